@@ -1,0 +1,205 @@
+/*
+ * autoverse.h -- C ABI of libautoverse.so, a batched GPU engine for the
+ * rewrite-rule game language of "Autoverse: an Evolvable Game Language for
+ * Learning Robust Embodied Agents" (Earle & Togelius, arXiv 2407.04221).
+ *
+ * Model (Sec. 2.1): a board is an H x W grid of multi-hot cells; bit c of a
+ * cell is tile channel c (c < C).  A rewrite rule is an input pattern, an
+ * output pattern and a reward (Sec. 2.1, Fig. 2a caption): where the input
+ * pattern is present at step t, the output pattern is written at t+1
+ * (Sec. 2.1, per-patch definition C_{t+1} = O if the input is present, else
+ * C_t), and the rule's reward is paid once per match (Sec. 2.2.1).  All rules
+ * apply in parallel to the same board (Sec. 2.1, end of "Possible
+ * extensions").  The player acts by placing an invisible force tile next to
+ * itself (Sec. 2.1, movement paragraph); force is channel C, visible to rules
+ * during the step and never stored.
+ *
+ * Fixed readings where the paper is silent:
+ *  - each rule is matched in 4 rotations (0/90/180/270 degrees CCW: entry
+ *    (i,k) of an h x w pattern goes to (w-1-k, i)); every (rule, rotation,
+ *    anchor) match counts and pays once;
+ *  - only VALID anchors (window fully inside the board);
+ *  - conflicting writes: a bit changes when any match asks it to:
+ *        next = (F & ~CLR) | (~F & SET), with F the board plus force;
+ *  - actions: 0 no-op, 1 up (-y), 2 right (+x), 3 down (+y), 4 left (-x);
+ *    values >= 5 act as no-op and raise AV_WARN_ACTION;
+ *  - done: no goal tile left (when ch_goal >= 0) or t >= max_steps (when
+ *    max_steps > 0); with auto_reset the env returns its own initial map
+ *    and t = 0; the observation returned is the board after any reset.
+ *
+ * Conventions.  Every function returns an int status (AV_OK = 0, negative on
+ * error) and never aborts.  Argument checks happen on the host before any
+ * launch (AV_EINVAL).  All pointers except av_config, av_rule and init_cum
+ * are CALLER-OWNED DEVICE pointers (may be NULL only where stated); work is
+ * enqueued on `stream` (a cudaStream_t cast to uintptr_t; 0 = legacy default
+ * stream) and returns without synchronising.  Asynchronous CUDA errors are
+ * reported by the next call that synchronises (av_sync, av_get_state with a
+ * host copy, or any call whose launch fails) as AV_ECUDA; av_last_error()
+ * gives the message.  A handle is not thread-safe.
+ *
+ * Board layout in memory ("canonical"): [H][W] cell words, row-major, each
+ * cell uint8_t when C <= 8, else uint16_t (little-endian), tile bits only.
+ * Batched boards are [B][H][W].
+ */
+#ifndef AUTOVERSE_H
+#define AUTOVERSE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    AV_OK = 0,
+    AV_EINVAL = -1,  /* bad argument, checked before any launch            */
+    AV_ENOMEM = -2,  /* device or host allocation failed                   */
+    AV_ECUDA = -3,   /* CUDA launch or runtime error                       */
+    AV_ESTATE = -4,  /* call not valid in the handle's state               */
+    AV_EDEVICE = -5  /* a kernel reported an error through its status word */
+};
+
+/* warning bits reported by av_warnings() */
+enum { AV_WARN_ACTION = 1 /* an action value >= 5 was treated as no-op */ };
+
+#define AV_MAX_SIDE 64   /* H, W <= 64                                   */
+#define AV_MAX_C 16      /* C <= 16 tile channels (+1 force channel)     */
+#define AV_MAX_PATTERN 5 /* rule patterns up to 5 x 5                    */
+#define AV_MAX_RULES 64  /* rules per table                              */
+
+typedef struct av_handle av_handle; /* opaque; owns all env state on the device */
+
+/* Configuration, copied by av_create. */
+typedef struct {
+    int32_t batch;         /* B >= 1 environments                                   */
+    int32_t H, W;          /* 1..AV_MAX_SIDE                                        */
+    int32_t C;             /* 1..AV_MAX_C tile channels; force is channel C         */
+    int32_t n_rules;       /* R rules per table, 0..AV_MAX_RULES                    */
+    int32_t rules_per_env; /* 1: rules[B][R]; 0: one table rules[R] for all envs    */
+    int32_t max_steps;     /* 0 = no step limit                                     */
+    int32_t auto_reset;    /* 1: a done env restores its initial map, t = 0         */
+    int32_t ch_player, ch_goal, ch_empty, ch_wall; /* role channels, -1 = none      */
+    int32_t border_wall;   /* av_reset: border cells hold only the wall tile        */
+    int32_t cum_per_env;   /* 1: init_cum[B][C]; 0: init_cum[C]                     */
+    const uint32_t *init_cum; /* HOST pointer, av_reset thresholds: a cell draws u in
+                                 [0, 2^24) and takes the first type t with u < cum[t];
+                                 copied by av_create; may be NULL (no av_reset)     */
+    int32_t search_capacity;  /* av_select: visited hashes kept per env (0 = none)  */
+} av_config;
+
+/* Packed rewrite rule, 408 bytes, little-endian (Sec. 2.1: input pattern I,
+ * output pattern O, reward).  Entry (i,k) of the h x w base pattern is index
+ * i*w + k.  present/absent: bit c (c <= C, bit C = force) must be 1 / 0 at
+ * that entry for a match; set/clear: bit c (c < C) written at t+1. */
+typedef struct {
+    uint8_t h, w;      /* 1..AV_MAX_PATTERN */
+    uint8_t _pad[2];
+    int32_t reward;    /* paid once per match */
+    uint32_t present[25], absent[25], set[25], clear[25];
+} av_rule;
+
+/* Create a handle: validates cfg and rules (HOST pointers: rules[B][R] or
+ * rules[R] per cfg->rules_per_env), compiles every rule in its 4 rotations
+ * and allocates the device state (current boards, initial boards, step
+ * counters t, compiled rules).  Boards start all-zero with t = 0 and are
+ * their own initial maps until av_reset or av_set_state(set_as_init=1).
+ * Returns AV_EINVAL for out-of-range fields, AV_ENOMEM, AV_ECUDA. */
+int av_create(const av_config *cfg, const av_rule *rules, av_handle **out);
+
+/* Release the handle and its device memory (after pending work finishes).
+ * A NULL handle is AV_EINVAL. */
+int av_destroy(av_handle *h);
+
+/* Draw every env's initial map from `seed` (stream 1: cell types from
+ * init_cum; stream 2: one player on a uniformly chosen floor cell, or on
+ * any interior cell when there is no floor), store it as both the current
+ * and the initial map, set t = 0.  obs: device [B][H][W] copy of the maps,
+ * or NULL.  AV_ESTATE if the handle has no init_cum. */
+int av_reset(av_handle *h, uint64_t seed, void *obs, uintptr_t stream);
+
+/* Replace the current boards (device [B][H][W]); t: device int32[B] or NULL
+ * (then t = 0); set_as_init = 1 also makes them the initial maps. */
+int av_set_state(av_handle *h, const void *grids, const int32_t *t, int set_as_init,
+                 uintptr_t stream);
+
+/* Copy the current boards to device [B][H][W] (and t to device int32[B]
+ * when t is not NULL). */
+int av_get_state(av_handle *h, void *grids, int32_t *t, uintptr_t stream);
+
+/* One batched step (Sec. 2.1): actions device uint8[B]; obs device
+ * [B][H][W] or NULL; reward device int32[B]; done device uint8[B] (reward
+ * and done may be NULL).  Updates the handle's boards and t. */
+int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, uint8_t *done,
+            uintptr_t stream);
+
+/* n_steps fused steps in one launch, boards held on chip.  The action of env
+ * b at step s (0-based within this call) is
+ *     a = ((draw(action_seed, 4, b, 0, s) >> 32) * 5) >> 32
+ * with draw the SplitMix64-keyed counter draw
+ *     draw(seed, st, a, b, c) = mix(mix(mix(seed + 0x9E3779B97F4A7C15*(st+1)) ^ a) ^ (b<<32|c)).
+ * Optional device outputs (NULL to skip): obs_traj [n_steps][B][H][W],
+ * rew_traj int32[n_steps][B], done_traj uint8[n_steps][B], rew_sum int32[B]
+ * (sum of this call's rewards). */
+int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_traj,
+               int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uintptr_t stream);
+
+/* Tree-search expansion (Sec. 2.2.1: the environment is its own forward
+ * model for best-first search over player actions): every parent board
+ * parents[b][f] (device [B][F][H][W]) stepped by each of the 5 actions with
+ * env b's rules -> children [B][F][5][H][W], rewards int32[B][F][5], done
+ * uint8[B][F][5] (no goal left; may be NULL) and hashes uint64[B][F][5]
+ * (FNV-1a 64 of the child's canonical bytes: offset basis
+ * 0xcbf29ce484222325, prime 0x100000001b3).  n_parent: device int32[B] or
+ * NULL; when given, parents f >= n_parent[b] are skipped and their output
+ * slots are left untouched.  No step counter, no reset: a child is the raw
+ * transition.  Stateless with respect to the handle's boards. */
+int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_parent,
+              void *children, int32_t *rewards, uint8_t *done, uint64_t *hashes,
+              uintptr_t stream);
+
+/* Start a search from the root boards roots (device [B][H][W]): writes
+ * root_hash uint64[B] (FNV-1a 64 as in av_expand) and root_live uint8[B]
+ * (1 unless the root has no goal left), and sets the visited set of env b
+ * to { root_hash[b] }.  AV_ESTATE if cfg.search_capacity < 1. */
+int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t *root_live,
+                   uintptr_t stream);
+
+/* One selection step of greedy best-first search (Sec. 2.2.1: states equal
+ * to an earlier one are pruned, keeping the shallower; of equal states the
+ * higher reward is kept).  Candidates are the children of av_expand for F
+ * parents per env: cand_grids [B][F][5][H][W], cand_reward int32[B][F][5],
+ * cand_done uint8[B][F][5], cand_hash uint64[B][F][5]; parent_cum int32[B][F]
+ * and parent_live uint8[B][F] (a candidate exists only for parent f <
+ * n_parent[b] with parent_live != 0; n_parent int32[B]).  Per env:
+ * cum = parent_cum + reward; drop hashes already visited; among equal
+ * hashes keep the highest cum (then the lowest candidate index); rank by
+ * (cum desc, hash asc); keep the first min(k, count) as the next frontier
+ * next_grids [B][k][H][W], next_cum int32[B][k], next_hash uint64[B][k],
+ * next_live uint8[B][k] (= !done), n_next int32[B]; add their hashes to the
+ * visited set.  AV_EINVAL if 5*F > 4096 or k > 5*F; AV_EDEVICE (via
+ * av_sync) if a visited set would exceed search_capacity. */
+int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *parent_cum,
+              const uint8_t *parent_live, const void *cand_grids, const int32_t *cand_reward,
+              const uint8_t *cand_done, const uint64_t *cand_hash, int32_t k, void *next_grids,
+              int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live, int32_t *n_next,
+              uintptr_t stream);
+
+/* Wait for the handle's pending work (device-wide synchronise) and report
+ * deferred errors: AV_ECUDA for a CUDA error, AV_EDEVICE when a kernel set
+ * its error status (e.g. visited set overflow). */
+int av_sync(av_handle *h);
+
+/* Warning bits seen since the last call (synchronises); see AV_WARN_*. */
+int av_warnings(av_handle *h, uint32_t *bits);
+
+/* Static description of a status code. */
+const char *av_strerror(int status);
+
+/* Message of the handle's last error ("" if none); valid until the next call. */
+const char *av_last_error(av_handle *h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AUTOVERSE_H */

@@ -1,0 +1,544 @@
+// autoverse.cu -- libautoverse.so: batched rewrite-rule engine for sm_103a.
+//
+// Host side: argument checks, rule compilation (every rule in its four
+// rotations, turned into term lists over bit-planes), device buffers, launches.
+// Device side: see kernels.cuh.
+//
+// Rule semantics follow Sec. 2.1 of Earle & Togelius, "Autoverse" (arXiv
+// 2407.04221): the per-patch rule definition, the matching convolution
+// ReLU(conv_{K_I}(D) - I + 1), the transposed-convolution write of the output
+// pattern, force tiles for actions, and parallel application of all rules.
+#include "autoverse.h"
+
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "kernels.cuh"
+
+using namespace av;
+
+struct av_handle {
+    DevConfig cf{};
+    av_config host_cfg{};
+    int n_tables = 0;
+    size_t grid_bytes = 0;  // one board, canonical bytes
+    // device buffers
+    uint32_t *d_arena = nullptr;
+    uint32_t *d_tab_off = nullptr;
+    uint32_t *d_vm = nullptr;
+    void *d_cur = nullptr;
+    void *d_init = nullptr;
+    int32_t *d_t = nullptr;
+    uint32_t *d_cum = nullptr;
+    uint32_t *d_status = nullptr;  // [0] error bits, [1] warning bits
+    uint64_t *d_visited = nullptr;  // [2][B][capacity] sorted hashes (double-buffered)
+    int32_t *d_n_visited = nullptr; // [B]
+    int vis_parity = 0;
+    bool has_cum = false;
+    std::string last_error;
+};
+
+namespace {
+
+int fail(av_handle *h, int code, const std::string &msg)
+{
+    if (h)
+        h->last_error = msg;
+    return code;
+}
+
+int cuda_fail(av_handle *h, cudaError_t e, const char *where)
+{
+    return fail(h, AV_ECUDA, std::string(where) + ": " + cudaGetErrorString(e));
+}
+
+#define AV_CUDA(h, call)                                                                   \
+    do {                                                                                   \
+        cudaError_t e_ = (call);                                                           \
+        if (e_ != cudaSuccess)                                                             \
+            return cuda_fail((h), e_, #call);                                              \
+    } while (0)
+
+// A rule pattern as the compiler sees it (base or rotated).
+struct Pat {
+    int h = 0, w = 0;
+    int32_t reward = 0;
+    uint32_t pres[25] = {}, abs_[25] = {}, set[25] = {}, clr[25] = {};
+};
+
+Pat from_record(const av_rule &r)
+{
+    Pat p;
+    p.h = r.h;
+    p.w = r.w;
+    p.reward = r.reward;
+    for (int e = 0; e < 25; ++e) {
+        p.pres[e] = r.present[e];
+        p.abs_[e] = r.absent[e];
+        p.set[e] = r.set[e];
+        p.clr[e] = r.clear[e];
+    }
+    return p;
+}
+
+// One counter-clockwise quarter turn: (i, k) of h x w -> (w-1-k, i) of w x h.
+Pat quarter_turn(const Pat &in)
+{
+    Pat out;
+    out.h = in.w;
+    out.w = in.h;
+    out.reward = in.reward;
+    for (int i = 0; i < in.h; ++i)
+        for (int k = 0; k < in.w; ++k) {
+            const int from = i * in.w + k;
+            const int to = (in.w - 1 - k) * out.w + i;
+            out.pres[to] = in.pres[from];
+            out.abs_[to] = in.abs_[from];
+            out.set[to] = in.set[from];
+            out.clr[to] = in.clr[from];
+        }
+    return out;
+}
+
+int check_config(const av_config *c, std::string &why)
+{
+    auto bad = [&](const char *m) { why = m; return AV_EINVAL; };
+    if (c->batch < 1) return bad("batch must be >= 1");
+    if (c->H < 1 || c->H > AV_MAX_SIDE || c->W < 1 || c->W > AV_MAX_SIDE) return bad("H, W must be in 1..64");
+    if (c->C < 1 || c->C > AV_MAX_C) return bad("C must be in 1..16");
+    if (c->n_rules < 0 || c->n_rules > AV_MAX_RULES) return bad("n_rules must be in 0..64");
+    if (c->rules_per_env != 0 && c->rules_per_env != 1) return bad("rules_per_env must be 0 or 1");
+    if (c->cum_per_env != 0 && c->cum_per_env != 1) return bad("cum_per_env must be 0 or 1");
+    if (c->max_steps < 0) return bad("max_steps must be >= 0");
+    if (c->auto_reset != 0 && c->auto_reset != 1) return bad("auto_reset must be 0 or 1");
+    if (c->search_capacity < 0) return bad("search_capacity must be >= 0");
+    const int32_t roles[4] = {c->ch_player, c->ch_goal, c->ch_empty, c->ch_wall};
+    for (int r : roles)
+        if (r < -1 || r >= c->C) return bad("role channels must be -1 or in 0..C-1");
+    return AV_OK;
+}
+
+int check_rule(const av_rule &r, int C, std::string &why)
+{
+    if (r.h < 1 || r.h > AV_MAX_PATTERN || r.w < 1 || r.w > AV_MAX_PATTERN) {
+        why = "rule h, w must be in 1..5";
+        return AV_EINVAL;
+    }
+    const uint32_t in_ok = (C + 1 >= 32) ? 0xffffffffu : ((1u << (C + 1)) - 1u);
+    const uint32_t out_ok = (1u << C) - 1u;
+    for (int e = 0; e < 25; ++e) {
+        const bool inside = e < r.h * r.w;
+        if ((r.present[e] | r.absent[e]) & ~(inside ? in_ok : 0u)) {
+            why = "rule input bits outside channels 0..C or outside the h x w pattern";
+            return AV_EINVAL;
+        }
+        if ((r.set[e] | r.clear[e]) & ~(inside ? out_ok : 0u)) {
+            why = "rule output bits outside channels 0..C-1 or outside the h x w pattern";
+            return AV_EINVAL;
+        }
+    }
+    return AV_OK;
+}
+
+// Compile one rule table into the arena format read by the kernels
+// (kernels.cuh, "rule table layout").
+void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32_t> &arena)
+{
+    const size_t base = arena.size();
+    const int K = 4 * cf.R;
+    std::vector<uint32_t> hdr(8 * (size_t)K, 0), items, terms, outs;
+    for (int r = 0; r < cf.R; ++r) {
+        Pat p = from_record(rules[r]);
+        for (int j = 0; j < 4; ++j, p = quarter_turn(p)) {
+            const int rr = 4 * r + j;
+            uint32_t *hd = &hdr[8 * (size_t)rr];
+            hd[0] = (uint32_t)((p.h - 1) * AV_MAX_PATTERN + (p.w - 1));
+            hd[3] = (uint32_t)p.reward;
+            hd[4] = (uint32_t)terms.size();
+            hd[5] = (uint32_t)(outs.size() / 2);
+            // terms: present before absent, force channel first, then channels descending
+            struct T { int neg, c, s; };
+            std::vector<T> ts;
+            for (int i = 0; i < p.h; ++i)
+                for (int k = 0; k < p.w; ++k) {
+                    const int e = i * p.w + k, s = i * cf.W + k;
+                    for (int c = 0; c <= cf.C; ++c) {
+                        if ((p.pres[e] >> c) & 1u) ts.push_back({0, c, s});
+                        if ((p.abs_[e] >> c) & 1u) ts.push_back({1, c, s});
+                    }
+                }
+            std::stable_sort(ts.begin(), ts.end(), [](const T &a, const T &b) {
+                if (a.neg != b.neg) return a.neg < b.neg;
+                return a.c > b.c;
+            });
+            for (const T &t : ts)
+                terms.push_back(encode_term(t.c, t.s, t.neg, cf.pstride));
+            hd[1] = (uint32_t)ts.size();
+            int no = 0;
+            for (int i = 0; i < p.h; ++i)
+                for (int k = 0; k < p.w; ++k) {
+                    const int e = i * p.w + k;
+                    if (p.set[e] | p.clr[e]) {
+                        outs.push_back((uint32_t)(i * cf.W + k));
+                        outs.push_back(p.set[e] | (p.clr[e] << 16));
+                        ++no;
+                    }
+                }
+            hd[2] = (uint32_t)no;
+            if (p.h <= cf.H && p.w <= cf.W) {
+                const int last = ((cf.H - p.h) * cf.W + (cf.W - p.w)) >> 5;
+                for (int a = 0; a <= last; ++a)
+                    items.push_back(((uint32_t)rr << 16) | (uint32_t)a);
+            }
+        }
+    }
+    const uint32_t items_off = 8 + 8 * (uint32_t)K;
+    const uint32_t terms_off = items_off + (uint32_t)items.size();
+    uint32_t outs_off = terms_off + (uint32_t)terms.size();
+    outs_off += outs_off & 1u;  // uint2 alignment
+    arena.resize(base + outs_off + outs.size(), 0);
+    uint32_t *t = &arena[base];
+    t[0] = (uint32_t)K;
+    t[1] = (uint32_t)items.size();
+    t[2] = items_off;
+    t[3] = terms_off;
+    t[4] = outs_off;
+    std::copy(hdr.begin(), hdr.end(), t + 8);
+    std::copy(items.begin(), items.end(), t + items_off);
+    std::copy(terms.begin(), terms.end(), t + terms_off);
+    std::copy(outs.begin(), outs.end(), t + outs_off);
+    while (arena.size() & 3u) arena.push_back(0);  // next table starts 16-byte aligned
+}
+
+// Valid-anchor masks: vm[shape][word] bit b set when anchor p = 32*word + b
+// has its h' x w' window inside the board.
+std::vector<uint32_t> valid_masks(const DevConfig &cf)
+{
+    std::vector<uint32_t> vm((size_t)AV_MAX_PATTERN * AV_MAX_PATTERN * cf.NW, 0);
+    for (int hh = 1; hh <= AV_MAX_PATTERN; ++hh)
+        for (int ww = 1; ww <= AV_MAX_PATTERN; ++ww) {
+            const int shape = (hh - 1) * AV_MAX_PATTERN + (ww - 1);
+            for (int p = 0; p < cf.HW; ++p) {
+                const int y = p / cf.W, x = p % cf.W;
+                if (y <= cf.H - hh && x <= cf.W - ww)
+                    vm[(size_t)shape * cf.NW + (p >> 5)] |= 1u << (p & 31);
+            }
+        }
+    return vm;
+}
+
+template <typename T>
+int dalloc(av_handle *h, T **p, size_t n)
+{
+    if (getenv("AV_FAIL_ALLOC"))  // host-side fault injection for the ENOMEM path
+        return fail(h, AV_ENOMEM, "allocation refused (AV_FAIL_ALLOC set)");
+    cudaError_t e = cudaMalloc((void **)p, n * sizeof(T) + (n == 0 ? 8 : 0));
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(h, e == cudaErrorMemoryAllocation ? AV_ENOMEM : AV_ECUDA,
+                    std::string("cudaMalloc: ") + cudaGetErrorString(e));
+    }
+    return AV_OK;
+}
+
+void free_all(av_handle *h)
+{
+    cudaFree(h->d_arena);
+    cudaFree(h->d_tab_off);
+    cudaFree(h->d_vm);
+    cudaFree(h->d_cur);
+    cudaFree(h->d_init);
+    cudaFree(h->d_t);
+    cudaFree(h->d_cum);
+    cudaFree(h->d_status);
+    cudaFree(h->d_visited);
+    cudaFree(h->d_n_visited);
+}
+
+cudaStream_t as_stream(uintptr_t s) { return reinterpret_cast<cudaStream_t>(s); }
+
+int launch_check(av_handle *h, const char *what)
+{
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return cuda_fail(h, e, what);
+    return AV_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------- C ABI
+extern "C" {
+
+const char *av_strerror(int s)
+{
+    switch (s) {
+    case AV_OK: return "ok";
+    case AV_EINVAL: return "invalid argument";
+    case AV_ENOMEM: return "out of memory";
+    case AV_ECUDA: return "CUDA error";
+    case AV_ESTATE: return "invalid handle state";
+    case AV_EDEVICE: return "device-side error";
+    default: return "unknown status";
+    }
+}
+
+const char *av_last_error(av_handle *h) { return h ? h->last_error.c_str() : "null handle"; }
+
+int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
+{
+    if (!cfg || !out || (cfg->n_rules > 0 && !rules))
+        return AV_EINVAL;
+    *out = nullptr;
+    std::string why;
+    if (check_config(cfg, why) != AV_OK)
+        return AV_EINVAL;
+    const int n_tables = cfg->rules_per_env ? cfg->batch : 1;
+    for (size_t i = 0; i < (size_t)n_tables * cfg->n_rules; ++i)
+        if (check_rule(rules[i], cfg->C, why) != AV_OK)
+            return AV_EINVAL;
+
+    av_handle *h = new (std::nothrow) av_handle();
+    if (!h)
+        return AV_ENOMEM;
+    h->host_cfg = *cfg;
+    h->host_cfg.init_cum = nullptr;
+    h->n_tables = n_tables;
+    DevConfig &cf = h->cf;
+    cf.B = cfg->batch;
+    cf.H = cfg->H;
+    cf.W = cfg->W;
+    cf.C = cfg->C;
+    cf.HW = cfg->H * cfg->W;
+    cf.NW = (cf.HW + 31) / 32;
+    cf.NWP = cf.NW + kPlanePad;
+    cf.pstride = cf.NWP * 8;
+    cf.R = cfg->n_rules;
+    cf.rules_per_env = cfg->rules_per_env;
+    cf.max_steps = cfg->max_steps;
+    cf.auto_reset = cfg->auto_reset;
+    cf.ch_player = cfg->ch_player;
+    cf.ch_goal = cfg->ch_goal;
+    cf.ch_empty = cfg->ch_empty;
+    cf.ch_wall = cfg->ch_wall;
+    cf.border_wall = cfg->border_wall ? 1 : 0;
+    cf.cum_per_env = cfg->cum_per_env;
+    cf.cell_bytes = cfg->C <= 8 ? 1 : 2;
+    h->grid_bytes = (size_t)cf.HW * cf.cell_bytes;
+
+    std::vector<uint32_t> arena, tab_off((size_t)n_tables);
+    for (int t = 0; t < n_tables; ++t) {
+        tab_off[t] = (uint32_t)arena.size();
+        compile_table(rules + (size_t)t * cfg->n_rules, cf, arena);
+    }
+    std::vector<uint32_t> vm = valid_masks(cf);
+
+    int rc;
+    const size_t B = (size_t)cf.B;
+    if ((rc = dalloc(h, &h->d_arena, arena.size())) || (rc = dalloc(h, &h->d_tab_off, tab_off.size())) ||
+        (rc = dalloc(h, &h->d_vm, vm.size())) ||
+        (rc = dalloc(h, (uint8_t **)&h->d_cur, B * h->grid_bytes)) ||
+        (rc = dalloc(h, (uint8_t **)&h->d_init, B * h->grid_bytes)) || (rc = dalloc(h, &h->d_t, B)) ||
+        (rc = dalloc(h, &h->d_status, 4))) {
+        free_all(h);
+        delete h;
+        return rc;
+    }
+    if (cfg->init_cum) {
+        const size_t ncum = (size_t)(cfg->cum_per_env ? cf.B : 1) * cf.C;
+        if ((rc = dalloc(h, &h->d_cum, ncum)) ||
+            cudaMemcpy(h->d_cum, cfg->init_cum, ncum * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
+            free_all(h);
+            delete h;
+            return rc ? rc : AV_ECUDA;
+        }
+        h->has_cum = true;
+    }
+    if (cfg->search_capacity > 0) {
+        if ((rc = dalloc(h, &h->d_visited, 2 * B * (size_t)cfg->search_capacity)) ||
+            (rc = dalloc(h, &h->d_n_visited, B))) {
+            free_all(h);
+            delete h;
+            return rc;
+        }
+        cudaMemset(h->d_n_visited, 0, B * 4);
+    }
+    cudaError_t e = cudaSuccess;
+    if (e == cudaSuccess) e = cudaMemcpy(h->d_arena, arena.data(), arena.size() * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(h->d_tab_off, tab_off.data(), tab_off.size() * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(h->d_vm, vm.data(), vm.size() * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemset(h->d_cur, 0, B * h->grid_bytes);
+    if (e == cudaSuccess) e = cudaMemset(h->d_init, 0, B * h->grid_bytes);
+    if (e == cudaSuccess) e = cudaMemset(h->d_t, 0, B * 4);
+    if (e == cudaSuccess) e = cudaMemset(h->d_status, 0, 16);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        free_all(h);
+        delete h;
+        return AV_ECUDA;
+    }
+    if (configure_kernels(cf) != cudaSuccess) {
+        free_all(h);
+        delete h;
+        return AV_ECUDA;
+    }
+    *out = h;
+    return AV_OK;
+}
+
+int av_destroy(av_handle *h)
+{
+    if (!h)
+        return AV_EINVAL;
+    cudaDeviceSynchronize();
+    free_all(h);
+    delete h;
+    return AV_OK;
+}
+
+int av_reset(av_handle *h, uint64_t seed, void *obs, uintptr_t stream)
+{
+    if (!h)
+        return AV_EINVAL;
+    if (!h->has_cum)
+        return fail(h, AV_ESTATE, "av_reset: the handle was created without init_cum");
+    launch_reset(h->cf, h->d_cum, seed, h->d_cur, h->d_init, h->d_t, obs, as_stream(stream));
+    return launch_check(h, "reset kernel");
+}
+
+int av_set_state(av_handle *h, const void *grids, const int32_t *t, int set_as_init, uintptr_t stream)
+{
+    if (!h || !grids)
+        return AV_EINVAL;
+    cudaStream_t s = as_stream(stream);
+    const size_t n = (size_t)h->cf.B * h->grid_bytes;
+    AV_CUDA(h, cudaMemcpyAsync(h->d_cur, grids, n, cudaMemcpyDeviceToDevice, s));
+    if (set_as_init)
+        AV_CUDA(h, cudaMemcpyAsync(h->d_init, grids, n, cudaMemcpyDeviceToDevice, s));
+    if (t)
+        AV_CUDA(h, cudaMemcpyAsync(h->d_t, t, (size_t)h->cf.B * 4, cudaMemcpyDeviceToDevice, s));
+    else
+        AV_CUDA(h, cudaMemsetAsync(h->d_t, 0, (size_t)h->cf.B * 4, s));
+    return AV_OK;
+}
+
+int av_get_state(av_handle *h, void *grids, int32_t *t, uintptr_t stream)
+{
+    if (!h || !grids)
+        return AV_EINVAL;
+    cudaStream_t s = as_stream(stream);
+    AV_CUDA(h, cudaMemcpyAsync(grids, h->d_cur, (size_t)h->cf.B * h->grid_bytes,
+                               cudaMemcpyDeviceToDevice, s));
+    if (t)
+        AV_CUDA(h, cudaMemcpyAsync(t, h->d_t, (size_t)h->cf.B * 4, cudaMemcpyDeviceToDevice, s));
+    return AV_OK;
+}
+
+int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, uint8_t *done,
+            uintptr_t stream)
+{
+    if (!h || !actions)
+        return AV_EINVAL;
+    launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_cur, h->d_init, h->d_t, 1, 0,
+                   actions, obs, reward, done, nullptr, h->d_status, as_stream(stream));
+    return launch_check(h, "step kernel");
+}
+
+int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_traj,
+               int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uintptr_t stream)
+{
+    if (!h || n_steps < 0)
+        return AV_EINVAL;
+    if (n_steps == 0)
+        return AV_OK;
+    launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_cur, h->d_init, h->d_t, n_steps,
+                   action_seed, nullptr, obs_traj, rew_traj, done_traj, rew_sum, h->d_status,
+                   as_stream(stream));
+    return launch_check(h, "rollout kernel");
+}
+
+int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_parent,
+              void *children, int32_t *rewards, uint8_t *done, uint64_t *hashes,
+              uintptr_t stream)
+{
+    if (!h || F < 0 || (F > 0 && (!parents || !children || !rewards || !hashes)))
+        return AV_EINVAL;
+    if ((size_t)h->cf.B * (size_t)F > 0x7fffffffu)
+        return AV_EINVAL;
+    if (F == 0)
+        return AV_OK;
+    launch_expand(h->cf, h->d_arena, h->d_tab_off, h->d_vm, parents, F, n_parent, children, rewards,
+                  done, hashes, as_stream(stream));
+    return launch_check(h, "expand kernel");
+}
+
+int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t *root_live,
+                   uintptr_t stream)
+{
+    if (!h || !roots || !root_hash || !root_live)
+        return AV_EINVAL;
+    if (h->host_cfg.search_capacity < 1)
+        return fail(h, AV_ESTATE, "av_search_init: search_capacity is 0");
+    h->vis_parity = 0;
+    launch_search_init(h->cf, h->host_cfg.search_capacity, roots, root_hash, root_live, h->d_visited,
+                       h->d_n_visited, as_stream(stream));
+    return launch_check(h, "search init kernel");
+}
+
+int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *parent_cum,
+              const uint8_t *parent_live, const void *cand_grids, const int32_t *cand_reward,
+              const uint8_t *cand_done, const uint64_t *cand_hash, int32_t k, void *next_grids,
+              int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live, int32_t *n_next,
+              uintptr_t stream)
+{
+    if (!h)
+        return AV_EINVAL;
+    if (h->host_cfg.search_capacity < 1)
+        return fail(h, AV_ESTATE, "av_select: search_capacity is 0");
+    if (F < 1 || 5 * F > kMaxCand || k < 1 || k > 5 * F)
+        return fail(h, AV_EINVAL, "av_select: need 1 <= F, 5*F <= 4096, 1 <= k <= 5*F");
+    if (!n_parent || !parent_cum || !parent_live || !cand_grids || !cand_reward || !cand_done ||
+        !cand_hash || !next_grids || !next_cum || !next_hash || !next_live || !n_next)
+        return AV_EINVAL;
+    launch_select(h->cf, h->host_cfg.search_capacity, h->vis_parity, F, n_parent, parent_cum,
+                  parent_live, cand_grids, cand_reward, cand_done, cand_hash, k, next_grids,
+                  next_cum, next_hash, next_live, n_next, h->d_visited, h->d_n_visited,
+                  h->d_status, as_stream(stream));
+    h->vis_parity ^= 1;
+    return launch_check(h, "select kernel");
+}
+
+int av_sync(av_handle *h)
+{
+    if (!h)
+        return AV_EINVAL;
+    AV_CUDA(h, cudaDeviceSynchronize());
+    uint32_t st[2] = {0, 0};
+    AV_CUDA(h, cudaMemcpy(st, h->d_status, 8, cudaMemcpyDeviceToHost));
+    if (st[0]) {
+        char buf[96];
+        snprintf(buf, sizeof buf, "device status 0x%x (bit 0: visited-set overflow)", st[0]);
+        AV_CUDA(h, cudaMemset(h->d_status, 0, 4));
+        return fail(h, AV_EDEVICE, buf);
+    }
+    return AV_OK;
+}
+
+int av_warnings(av_handle *h, uint32_t *bits)
+{
+    if (!h || !bits)
+        return AV_EINVAL;
+    AV_CUDA(h, cudaDeviceSynchronize());
+    AV_CUDA(h, cudaMemcpy(bits, h->d_status + 1, 4, cudaMemcpyDeviceToHost));
+    AV_CUDA(h, cudaMemset(h->d_status + 1, 0, 4));
+    return AV_OK;
+}
+
+}  // extern "C"

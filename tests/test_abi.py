@@ -1,0 +1,92 @@
+"""The C-ABI library loads and exports every entry point its header declares.
+
+No compute call is made here (no GPU needed): only host-side argument checks
+that return before any CUDA work.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "autoverse.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:int|const char \*)\s*(av_\w+)\s*\(", text, flags=re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2407_04221_gb300 import build
+    build.build()
+    import paper_2407_04221_gb300 as av
+    return av.load()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for n in ("av_create", "av_destroy", "av_reset", "av_step", "av_rollout", "av_expand",
+              "av_select", "av_sync"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    import paper_2407_04221_gb300 as av
+    names = declared_functions()
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+    assert set(names) == set(av.EXPORTS)
+
+
+def test_rule_record_size_matches_header():
+    import workload as wk
+    assert wk.RULE_DTYPE.itemsize == 408
+    text = open(HEADER).read()
+    assert "uint32_t present[25], absent[25], set[25], clear[25];" in text
+
+
+def test_host_side_argument_checks(lib):
+    import paper_2407_04221_gb300 as av
+    assert lib.av_destroy(None) == av.AV_EINVAL
+    assert lib.av_sync(None) == av.AV_EINVAL
+    assert lib.av_create(None, None, None) == av.AV_EINVAL
+    assert av.av_strerror(av.AV_EINVAL) == "invalid argument"
+    base = dict(batch=1, H=16, W=16, C=4, n_rules=0, rules_per_env=0, max_steps=0, auto_reset=0,
+                ch_player=2, ch_goal=3, ch_empty=0, ch_wall=1, border_wall=1, cum_per_env=0)
+    bad = [dict(batch=0), dict(H=65), dict(W=0), dict(C=17), dict(C=0), dict(n_rules=65),
+           dict(ch_goal=4), dict(ch_player=-2), dict(rules_per_env=2), dict(max_steps=-1)]
+    for b in bad:
+        with pytest.raises(av.AvError) as ei:
+            av.av_create(dict(base, **b), np.zeros(0, np.uint8))
+        assert ei.value.status == av.AV_EINVAL, b
+    # malformed rule records are rejected before any device work
+    import workload as wk
+    r = wk.empty_rules(1, 1)
+    r["h"], r["w"] = 3, 3
+    r["present"][0, 0, 9] = 1  # entry outside the 3x3 window
+    with pytest.raises(av.AvError):
+        av.av_create(dict(base, n_rules=1), r)
+    r = wk.empty_rules(1, 1)
+    r["h"], r["w"] = 6, 1
+    with pytest.raises(av.AvError):
+        av.av_create(dict(base, n_rules=1), r)
+    r = wk.empty_rules(1, 1)
+    r["h"], r["w"] = 1, 1
+    r["set"][0, 0, 0] = 1 << 4  # writes the force channel
+    with pytest.raises(av.AvError):
+        av.av_create(dict(base, n_rules=1), r)
+
+
+def test_missing_library_fails_loudly(tmp_path, monkeypatch):
+    import paper_2407_04221_gb300 as av
+    monkeypatch.setattr(av, "_lib", None)
+    monkeypatch.setattr(av, "LIB_PATH", str(tmp_path / "absent.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        av.load()

@@ -249,11 +249,15 @@ def make_init_cum(wl: Workload, seed: int) -> np.ndarray:
 
 def config_fields(wl: Workload) -> dict:
     """Scalar fields of the library's / oracle's configuration structs."""
+    def role(ch):
+        return ch if ch < wl.C else -1
+
     return dict(
         batch=wl.batch, H=wl.H, W=wl.W, C=wl.C, n_rules=wl.n_rules,
         rules_per_env=wl.rules_per_env, max_steps=wl.max_steps, auto_reset=wl.auto_reset,
-        ch_player=CH_PLAYER, ch_goal=CH_GOAL, ch_empty=CH_EMPTY, ch_wall=CH_WALL,
-        border_wall=wl.border_wall, cum_per_env=0 if wl.init == "maze" else 1,
+        ch_player=role(CH_PLAYER), ch_goal=role(CH_GOAL), ch_empty=role(CH_EMPTY),
+        ch_wall=role(CH_WALL), border_wall=wl.border_wall,
+        cum_per_env=0 if wl.init == "maze" else 1,
     )
 
 
