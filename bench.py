@@ -1,0 +1,377 @@
+"""Benchmark: batched Autoverse environment steps on one GB300 (per process).
+
+Default workload: 1024 envs, 16x16 boards, 8 tile channels, 8 rules of 3x3 in
+4 rotations each, per-env rule tables, 1000 fused steps per launch
+(av_rollout).  One benchmark step = one launch = 1024 x 1000 env-steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--config 2|3|5] [--seed S]
+
+Prints one JSON line.  Under torchrun (N > 1) every rank runs its own replica
+of the workload (envs never interact: no data-path collective); the timing is
+the max over ranks and `value` counts the env-steps of all ranks.
+
+--impl reference times the CPU oracle (the slow, literal restatement of the
+paper's rule semantics) on this machine's host cores, on a bounded sample of
+the same workload; only rank 0 runs it.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workload as wk  # noqa: E402
+
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+KERNEL_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "kernels.cuh")
+PROFILE = os.path.join(ROOT, "profiles", "rollout_kernel_grid16_b1024.md")
+SM_COUNT_GB300 = 152
+INT_LANES_PER_SM = 64  # 32-bit integer logic/shift/add lanes per SM per clock (4 SMSPs x 16)
+
+
+# ------------------------------------------------------------ workload
+def workload_for(key: int) -> wk.Workload:
+    return wk.WORKLOADS[key]
+
+
+def algorithmic_ops(wl: wk.Workload, rules: np.ndarray) -> float:
+    """Full-evaluation 32-bit word ops for one env-step, averaged over envs.
+
+    Every rule rotation tests each of its input terms (a present or absent
+    (position, channel) entry) at each valid anchor, and ORs each of its
+    output entries (set or clear, per position and channel) at each valid
+    anchor: one 32-bit op handles 32 anchors.  Rotation keeps the term and
+    output counts; a 90-degree turn swaps h and w for the anchor count.
+    """
+    h = rules["h"].astype(np.int64)
+    w = rules["w"].astype(np.int64)
+
+    def popc(a):
+        a = a.astype(np.uint64)
+        c = np.zeros(a.shape, np.int64)
+        for b in range(32):
+            c += ((a >> np.uint64(b)) & np.uint64(1)).astype(np.int64)
+        return c
+
+    terms = popc(rules["present"]).sum(-1) + popc(rules["absent"]).sum(-1)
+    outs = popc(rules["set"]).sum(-1) + popc(rules["clear"]).sum(-1)
+    va = np.clip(wl.H - h + 1, 0, None) * np.clip(wl.W - w + 1, 0, None)
+    vb = np.clip(wl.H - w + 1, 0, None) * np.clip(wl.W - h + 1, 0, None)
+    anchors = 2 * va + 2 * vb  # rotations 0, 2 and 1, 3
+    per_table = ((terms + outs) * anchors).sum(-1) / 32.0
+    return float(per_table.mean())
+
+
+# --------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = [r.split(",") for r in out.strip().splitlines() if r.count(",") >= 8]
+        if not rows:
+            return None
+        mhz = [float(r[1]) for r in rows]
+        mx = max(float(r[2]) for r in rows)
+        reasons = set()
+        for r in rows:
+            for name, col in (("hw_slowdown", 5), ("hw_thermal_slowdown", 6),
+                              ("sw_thermal_slowdown", 7), ("sw_power_cap", 8)):
+                if r[col].strip().lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows)}
+
+
+# -------------------------------------------------------------- helpers
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks() -> dict:
+    try:
+        return json.load(open(PEAKS_FILE))
+    except (OSError, ValueError):
+        return {}
+
+
+def profile_traffic() -> float | None:
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source."""
+    try:
+        text = open(PROFILE).read()
+    except OSError:
+        return None
+    m = re.search(r"kernel_source_sha256:\s*([0-9a-f]{16,64})", text)
+    t = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not m or not t:
+        return None
+    cur = hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()
+    return float(t.group(1)) if cur.startswith(m.group(1)) else None
+
+
+def cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0) -> dict:
+    """The oracle as it stands, all host cores, on a bounded sample of envs."""
+    import oracle
+    threads = os.cpu_count() or 1
+    s = wk.seeds(seed)
+    n = max(threads, 8)
+    steps = wl.steps
+    while True:
+        ids = np.arange(n)
+        g = oracle.reset(cfg, cum, s["reset"], ids)
+        t0 = time.perf_counter()
+        oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), steps, s["actions"], env_ids=ids,
+                       threads=threads)
+        dt = time.perf_counter() - t0
+        if dt > budget_s / 4 or n >= wl.batch:
+            break
+        n = min(wl.batch, int(n * max(2.0, budget_s / 4 / max(dt, 1e-3))))
+    return {"value": n * steps / dt, "unit": "env-steps/s", "cores": threads, "kind": "oracle",
+            "sample": f"{n} of {wl.batch} envs x {steps} fused steps (envs are independent)",
+            "seconds": dt}
+
+
+# ------------------------------------------------------------ reference
+def run_reference(args, wl):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    _, rules, cum = wk.make(wl, args.seed)
+    fields = wk.config_fields(wl)
+    cfg = oracle.make_cfg(**fields)
+    threads = os.cpu_count() or 1
+    s = wk.seeds(args.seed)
+    n = max(threads, 16)
+    ids = np.arange(n)
+    g = oracle.reset(cfg, cum, s["reset"], ids)
+    for _ in range(args.warmup):
+        oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), 50, s["actions"], env_ids=ids,
+                       threads=threads)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), wl.steps, s["actions"],
+                       env_ids=ids, threads=threads)
+        times.append(time.perf_counter() - t0)
+    mean = sum(times) / len(times)
+    value = n * wl.steps / mean
+    line = {
+        "impl": "reference", "metric": "env-steps/s", "value": value, "unit": "env-steps/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+        "data": "synthetic", "config": config_dict(wl, sample=n),
+        "cpu_baseline": {"value": value, "unit": "env-steps/s", "cores": threads,
+                         "kind": "oracle",
+                         "sample": f"{n} of {wl.batch} envs x {wl.steps} fused steps per step"},
+        "e2e": {"value": value, "unit": "env-steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def config_dict(wl, sample=None):
+    d = {"workload": f"{wl.name} (BASELINE config {wl.key})", "batch": wl.batch, "H": wl.H,
+         "W": wl.W, "tile_channels": wl.C, "rules": wl.n_rules, "rotations": 4,
+         "pattern_sizes": [f"{h}x{w}" for h, w in wl.shapes],
+         "fused_steps_per_launch": wl.steps, "per_env_rules": bool(wl.rules_per_env),
+         "trajectory_outputs": wl.trajectory,
+         "l2": "flushed (256 MiB write) between timed launches", "parallelism": "replicas"}
+    if sample:
+        d["sample_envs"] = sample
+    return d
+
+
+# ------------------------------------------------------------------ ours
+def run_ours(args, wl):
+    import torch
+
+    import paper_2407_04221_gb300 as av
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    seed = args.seed + 1000 * rank
+    _, rules, cum = wk.make(wl, seed)
+    fields = wk.config_fields(wl)
+    env = av.Env(fields, rules, cum, device=dev)
+    s = wk.seeds(seed)
+    g0 = env.reset(s["reset"])
+    stream = torch.cuda.current_stream(dev)
+    traj = None
+    if wl.trajectory:
+        traj = (env.boards(wl.steps, wl.batch),
+                torch.zeros(wl.steps, wl.batch, dtype=torch.int32, device=dev),
+                torch.zeros(wl.steps, wl.batch, dtype=torch.uint8, device=dev))
+    rew_sum = torch.zeros(wl.batch, dtype=torch.int32, device=dev)
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+
+    def launch(i):
+        obs, rew, done = traj if traj else (None, None, None)
+        av.av_rollout(env.h, wl.steps, s["actions"] + 7919 * i, obs, rew, done, rew_sum, stream)
+
+    for i in range(args.warmup):
+        launch(i)
+    torch.cuda.synchronize(dev)
+    env.sync()
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(torch.cuda.current_device() if world == 1 else local)
+    sampler.start()
+    barrier()
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.fill_(i & 0xff)  # evict L2 between timed launches (outside the events)
+        starts[i].record(stream)
+        launch(args.warmup + i)
+        ends[i].record(stream)
+    barrier()
+    wall = time.perf_counter() - t_wall
+    clocks = sampler.stop()
+    env.sync()
+    ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
+    kernel_ms = sum(ms) / len(ms)
+    total_ms = sum(ms)
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    env_steps = wl.batch * wl.steps * args.steps * world
+    value = env_steps / (total_ms / 1e3)
+    cells_rules = wl.H * wl.W * wl.n_rules * 4
+
+    # ---- e2e: the same launch through host buffers (pinned), copies timed
+    host_in = g0.cpu().pin_memory()
+    host_out = torch.empty(wl.batch, dtype=torch.int32).pin_memory()
+    dev_in = torch.empty_like(g0)
+    e2e_steps = max(3, min(args.steps, 20))
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_steps):
+        dev_in.copy_(host_in, non_blocking=True)
+        av.av_set_state(env.h, dev_in, None, False, stream)
+        launch(10_000 + i)
+        host_out.copy_(rew_sum, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e_value = wl.batch * wl.steps * world / (e2e_ms / 1e3)
+
+    if rank == 0:
+        peaks = measured_peaks()
+        sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+        peak_ops = SM_COUNT_GB300 * INT_LANES_PER_SM * sm_max * 1e6 / 1e9  # Gop/s
+        ops = algorithmic_ops(wl, rules)
+        achieved = ops * wl.batch * wl.steps / (kernel_ms / 1e3) / 1e9
+        traffic = profile_traffic()
+        line = {
+            "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+            "data": "synthetic", "config": config_dict(wl),
+            "cell_rule_updates_per_s": value * cells_rules,
+            "e2e": {"value": e2e_value, "unit": "env-steps/s",
+                    "h2d_bytes_per_step": int(host_in.numel() * host_in.element_size()),
+                    "d2h_bytes_per_step": int(host_out.numel() * host_out.element_size())},
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": peak_ops,
+                         "unit": "Gop/s", "frac": achieved / peak_ops,
+                         "traffic": traffic,
+                         "kernel": "rollout_kernel<uint8_t>",
+                         "ops_per_env_step": ops,
+                         "peak_from": f"{SM_COUNT_GB300} SMs x {INT_LANES_PER_SM} int32 lanes/clk"
+                                      f" x {sm_max:.0f} MHz (sm_max_mhz of measured peaks)"},
+            "gpu_launches": args.steps,
+            "wall_s_timed_region": wall,
+        }
+        if clocks:
+            line["clocks"] = clocks
+        if world == 1 and not args.no_cpu_baseline:
+            import oracle
+            cfg = oracle.make_cfg(**fields)
+            line["cpu_baseline"] = cpu_baseline(wl, rules, cum, cfg, seed)
+        print(json.dumps(line))
+    env.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--config", type=int, default=2, choices=(2, 3, 5))
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    wl = workload_for(args.config)
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_ours(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

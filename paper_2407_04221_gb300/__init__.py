@@ -122,8 +122,11 @@ def av_create(cfg: dict, rules, init_cum=None, search_capacity: int = 0):
         if name not in ("init_cum", "search_capacity"):
             setattr(c, name, int(cfg[name]))
     c.search_capacity = int(search_capacity)
-    rb = np.ascontiguousarray(np.frombuffer(memoryview(np.ascontiguousarray(rules)).cast("B"),
-                                            dtype=np.uint8))
+    if isinstance(rules, (bytes, bytearray, memoryview)):
+        rb = np.frombuffer(rules, dtype=np.uint8)
+    else:
+        a = np.ascontiguousarray(rules)
+        rb = a.reshape(-1).view(np.uint8) if a.size else np.zeros(0, np.uint8)
     if rb.size % RULE_BYTES:
         raise ValueError("rules must be packed 408-byte records")
     cum = None

@@ -33,6 +33,7 @@ struct av_handle {
     uint32_t *d_arena = nullptr;
     uint32_t *d_tab_off = nullptr;
     uint32_t *d_vm = nullptr;
+    uint32_t *d_masks = nullptr;
     void *d_cur = nullptr;
     void *d_init = nullptr;
     int32_t *d_t = nullptr;
@@ -88,25 +89,6 @@ Pat from_record(const av_rule &r)
     return p;
 }
 
-// One counter-clockwise quarter turn: (i, k) of h x w -> (w-1-k, i) of w x h.
-Pat quarter_turn(const Pat &in)
-{
-    Pat out;
-    out.h = in.w;
-    out.w = in.h;
-    out.reward = in.reward;
-    for (int i = 0; i < in.h; ++i)
-        for (int k = 0; k < in.w; ++k) {
-            const int from = i * in.w + k;
-            const int to = (in.w - 1 - k) * out.w + i;
-            out.pres[to] = in.pres[from];
-            out.abs_[to] = in.abs_[from];
-            out.set[to] = in.set[from];
-            out.clr[to] = in.clr[from];
-        }
-    return out;
-}
-
 int check_config(const av_config *c, std::string &why)
 {
     auto bad = [&](const char *m) { why = m; return AV_EINVAL; };
@@ -147,81 +129,129 @@ int check_rule(const av_rule &r, int C, std::string &why)
     return AV_OK;
 }
 
-// Compile one rule table into the arena format read by the kernels
-// (kernels.cuh, "rule table layout").
+// Position (i, k) of an h x w pattern after g counter-clockwise quarter turns.
+void turn_position(int h, int w, int g, int &i, int &k)
+{
+    for (int q = 0; q < g; ++q) {
+        const int ni = w - 1 - k, nk = i;
+        i = ni;
+        k = nk;
+        const int t = h;
+        h = w;
+        w = t;
+    }
+}
+
+// Compile one rule table into the layout read by the kernels (kernels.cuh,
+// "Rule table layout").  The term order is chosen once on the base pattern
+// and carried through every rotation, so the four rotations of a rule run
+// the same loop: present entries first -- positions with more present
+// channels first (two present tile types at one cell rule each other out on
+// one-hot boards), then the force channel, the player channel, higher
+// channels -- and absent entries last.  Any order gives the same result.
 void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32_t> &arena)
 {
     const size_t base = arena.size();
-    const int K = 4 * cf.R;
-    std::vector<uint32_t> hdr(8 * (size_t)K, 0), items, terms, outs;
-    for (int r = 0; r < cf.R; ++r) {
-        Pat p = from_record(rules[r]);
-        for (int j = 0; j < 4; ++j, p = quarter_turn(p)) {
-            const int rr = 4 * r + j;
-            uint32_t *hd = &hdr[8 * (size_t)rr];
-            hd[0] = (uint32_t)((p.h - 1) * AV_MAX_PATTERN + (p.w - 1));
-            hd[3] = (uint32_t)p.reward;
-            hd[4] = (uint32_t)terms.size();
-            hd[5] = (uint32_t)(outs.size() / 2);
-            // terms: present before absent, force channel first, then channels descending
-            struct T { int neg, c, s; };
-            std::vector<T> ts;
-            for (int i = 0; i < p.h; ++i)
-                for (int k = 0; k < p.w; ++k) {
-                    const int e = i * p.w + k, s = i * cf.W + k;
-                    for (int c = 0; c <= cf.C; ++c) {
-                        if ((p.pres[e] >> c) & 1u) ts.push_back({0, c, s});
-                        if ((p.abs_[e] >> c) & 1u) ts.push_back({1, c, s});
-                    }
+    const int R = cf.R;
+    std::vector<uint32_t> hdr(8 * (size_t)R, 0), terms, outs;
+    uint32_t n_terms = 0, n_outs = 0;
+    for (int r = 0; r < R; ++r) {
+        const Pat p = from_record(rules[r]);
+        struct BT { int i, k, c, neg, key0, key1; };
+        std::vector<BT> pres, absn;
+        for (int i = 0; i < p.h; ++i)
+            for (int k = 0; k < p.w; ++k) {
+                const int e = i * p.w + k;
+                const int npos = __builtin_popcount(p.pres[e]);
+                for (int c = 0; c <= cf.C; ++c) {
+                    const int rank = c == cf.C ? 2 : (c == cf.ch_player ? 1 : 0);
+                    const int key0 = c == cf.C ? 100 + npos : npos;  // a present force term first
+                    if ((p.pres[e] >> c) & 1u) pres.push_back({i, k, c, 0, key0, rank});
+                    if ((p.abs_[e] >> c) & 1u) absn.push_back({i, k, c, 1, 0, 0});
                 }
-            std::stable_sort(ts.begin(), ts.end(), [](const T &a, const T &b) {
-                if (a.neg != b.neg) return a.neg < b.neg;
-                return a.c > b.c;
-            });
-            for (const T &t : ts)
-                terms.push_back(encode_term(t.c, t.s, t.neg, cf.pstride));
-            hd[1] = (uint32_t)ts.size();
-            int no = 0;
-            for (int i = 0; i < p.h; ++i)
-                for (int k = 0; k < p.w; ++k) {
-                    const int e = i * p.w + k;
-                    if (p.set[e] | p.clr[e]) {
-                        outs.push_back((uint32_t)(i * cf.W + k));
-                        outs.push_back(p.set[e] | (p.clr[e] << 16));
-                        ++no;
-                    }
-                }
-            hd[2] = (uint32_t)no;
-            if (p.h <= cf.H && p.w <= cf.W) {
-                const int last = ((cf.H - p.h) * cf.W + (cf.W - p.w)) >> 5;
-                for (int a = 0; a <= last; ++a)
-                    items.push_back(((uint32_t)rr << 16) | (uint32_t)a);
             }
+        std::stable_sort(pres.begin(), pres.end(), [](const BT &a, const BT &b) {
+            if (a.key0 != b.key0) return a.key0 > b.key0;
+            if (a.key0 > 1 && a.key0 < 100 && a.i * 8 + a.k != b.i * 8 + b.k)
+                return a.i * 8 + a.k < b.i * 8 + b.k;  // keep a position's present terms together
+            if (a.key1 != b.key1) return a.key1 > b.key1;
+            return a.c > b.c;
+        });
+        uint32_t *hd = &hdr[8 * (size_t)r];
+        hd[0] = (uint32_t)pres.size();
+        hd[1] = (uint32_t)absn.size();
+        hd[3] = (uint32_t)p.reward;
+        hd[4] = n_terms;
+        hd[5] = n_outs;
+        uint32_t shapes = 0;
+        for (int g = 0; g < 4; ++g) {
+            const int hh = (g & 1) ? p.w : p.h, ww = (g & 1) ? p.h : p.w;
+            shapes |= (uint32_t)((hh - 1) * AV_MAX_PATTERN + (ww - 1)) << (8 * g);
         }
+        hd[6] = shapes;
+        std::vector<BT> all(pres);
+        all.insert(all.end(), absn.begin(), absn.end());
+        for (const BT &t : all) {
+            for (int g = 0; g < 4; ++g) {
+                int i = t.i, k = t.k;
+                turn_position(p.h, p.w, g, i, k);
+                const int s = i * cf.W + k;
+                terms.push_back((uint32_t)((t.c * cf.NWP + (s >> 5)) * 8));
+                terms.push_back((uint32_t)(s & 31));
+            }
+            ++n_terms;
+        }
+        uint32_t no = 0;
+        for (int i0 = 0; i0 < p.h; ++i0)
+            for (int k0 = 0; k0 < p.w; ++k0) {
+                const int e = i0 * p.w + k0;
+                if (!(p.set[e] | p.clr[e]))
+                    continue;
+                for (int g = 0; g < 4; ++g) {
+                    int i = i0, k = k0;
+                    turn_position(p.h, p.w, g, i, k);
+                    const int s = i * cf.W + k;
+                    outs.push_back((uint32_t)(s >> 5));
+                    outs.push_back((uint32_t)(s & 31));
+                    outs.push_back(p.set[e]);
+                    outs.push_back(p.clr[e]);
+                }
+                ++no;
+            }
+        hd[2] = no;
+        n_outs += no;
     }
-    const uint32_t items_off = 8 + 8 * (uint32_t)K;
-    const uint32_t terms_off = items_off + (uint32_t)items.size();
-    uint32_t outs_off = terms_off + (uint32_t)terms.size();
-    outs_off += outs_off & 1u;  // uint2 alignment
-    arena.resize(base + outs_off + outs.size(), 0);
+    const uint32_t tw = table_terms_word(R), ow = table_outs_word(R, n_terms);
+    arena.resize(base + ow + outs.size(), 0);
     uint32_t *t = &arena[base];
-    t[0] = (uint32_t)K;
-    t[1] = (uint32_t)items.size();
-    t[2] = items_off;
-    t[3] = terms_off;
-    t[4] = outs_off;
-    std::copy(hdr.begin(), hdr.end(), t + 8);
-    std::copy(items.begin(), items.end(), t + items_off);
-    std::copy(terms.begin(), terms.end(), t + terms_off);
-    std::copy(outs.begin(), outs.end(), t + outs_off);
+    t[0] = (uint32_t)R;
+    t[1] = n_terms;
+    t[2] = n_outs;
+    std::copy(hdr.begin(), hdr.end(), t + 4);
+    std::copy(terms.begin(), terms.end(), t + tw);
+    std::copy(outs.begin(), outs.end(), t + ow);
     while (arena.size() & 3u) arena.push_back(0);  // next table starts 16-byte aligned
+}
+
+// Column and cell masks over plane words: first column, last column, cells < H*W.
+std::vector<uint32_t> column_masks(const DevConfig &cf)
+{
+    std::vector<uint32_t> m(3 * (size_t)cf.NW, 0);
+    for (int p = 0; p < cf.HW; ++p) {
+        const int x = p % cf.W, w = p >> 5;
+        const uint32_t bit = 1u << (p & 31);
+        if (x == 0) m[w] |= bit;
+        if (x == cf.W - 1) m[cf.NW + w] |= bit;
+        m[2 * cf.NW + w] |= bit;
+    }
+    return m;
 }
 
 // Valid-anchor masks: vm[shape][word] bit b set when anchor p = 32*word + b
 // has its h' x w' window inside the board.
 std::vector<uint32_t> valid_masks(const DevConfig &cf)
 {
-    std::vector<uint32_t> vm((size_t)AV_MAX_PATTERN * AV_MAX_PATTERN * cf.NW, 0);
+    std::vector<uint32_t> vm((size_t)kShapes * cf.NW, 0);
     for (int hh = 1; hh <= AV_MAX_PATTERN; ++hh)
         for (int ww = 1; ww <= AV_MAX_PATTERN; ++ww) {
             const int shape = (hh - 1) * AV_MAX_PATTERN + (ww - 1);
@@ -253,6 +283,7 @@ void free_all(av_handle *h)
     cudaFree(h->d_arena);
     cudaFree(h->d_tab_off);
     cudaFree(h->d_vm);
+    cudaFree(h->d_masks);
     cudaFree(h->d_cur);
     cudaFree(h->d_init);
     cudaFree(h->d_t);
@@ -318,8 +349,8 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     cf.C = cfg->C;
     cf.HW = cfg->H * cfg->W;
     cf.NW = (cf.HW + 31) / 32;
-    cf.NWP = cf.NW + kPlanePad;
-    cf.pstride = cf.NWP * 8;
+    cf.NA = anchor_slots(cf.NW);
+    cf.NWP = 8 * cf.NA + kPlanePad;
     cf.R = cfg->n_rules;
     cf.rules_per_env = cfg->rules_per_env;
     cf.max_steps = cfg->max_steps;
@@ -333,17 +364,22 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     cf.cell_bytes = cfg->C <= 8 ? 1 : 2;
     h->grid_bytes = (size_t)cf.HW * cf.cell_bytes;
 
-    std::vector<uint32_t> arena, tab_off((size_t)n_tables);
+    std::vector<uint32_t> arena, tab_off((size_t)n_tables + 1);
+    uint32_t max_words = 0;
     for (int t = 0; t < n_tables; ++t) {
         tab_off[t] = (uint32_t)arena.size();
         compile_table(rules + (size_t)t * cfg->n_rules, cf, arena);
+        max_words = std::max(max_words, (uint32_t)arena.size() - tab_off[t]);
     }
+    tab_off[n_tables] = (uint32_t)arena.size();
+    cf.rule_words = max_words <= (uint32_t)kMaxSmemRuleWords ? (int)max_words : 0;
     std::vector<uint32_t> vm = valid_masks(cf);
+    std::vector<uint32_t> masks = column_masks(cf);
 
     int rc;
     const size_t B = (size_t)cf.B;
     if ((rc = dalloc(h, &h->d_arena, arena.size())) || (rc = dalloc(h, &h->d_tab_off, tab_off.size())) ||
-        (rc = dalloc(h, &h->d_vm, vm.size())) ||
+        (rc = dalloc(h, &h->d_vm, vm.size())) || (rc = dalloc(h, &h->d_masks, masks.size())) ||
         (rc = dalloc(h, (uint8_t **)&h->d_cur, B * h->grid_bytes)) ||
         (rc = dalloc(h, (uint8_t **)&h->d_init, B * h->grid_bytes)) || (rc = dalloc(h, &h->d_t, B)) ||
         (rc = dalloc(h, &h->d_status, 4))) {
@@ -374,6 +410,7 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     if (e == cudaSuccess) e = cudaMemcpy(h->d_arena, arena.data(), arena.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(h->d_tab_off, tab_off.data(), tab_off.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(h->d_vm, vm.data(), vm.size() * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(h->d_masks, masks.data(), masks.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemset(h->d_cur, 0, B * h->grid_bytes);
     if (e == cudaSuccess) e = cudaMemset(h->d_init, 0, B * h->grid_bytes);
     if (e == cudaSuccess) e = cudaMemset(h->d_t, 0, B * 4);
@@ -446,7 +483,7 @@ int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, ui
 {
     if (!h || !actions)
         return AV_EINVAL;
-    launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_cur, h->d_init, h->d_t, 1, 0,
+    launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur, h->d_init, h->d_t, 1, 0,
                    actions, obs, reward, done, nullptr, h->d_status, as_stream(stream));
     return launch_check(h, "step kernel");
 }
@@ -458,7 +495,7 @@ int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_tr
         return AV_EINVAL;
     if (n_steps == 0)
         return AV_OK;
-    launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_cur, h->d_init, h->d_t, n_steps,
+    launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur, h->d_init, h->d_t, n_steps,
                    action_seed, nullptr, obs_traj, rew_traj, done_traj, rew_sum, h->d_status,
                    as_stream(stream));
     return launch_check(h, "rollout kernel");
@@ -474,7 +511,7 @@ int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_par
         return AV_EINVAL;
     if (F == 0)
         return AV_OK;
-    launch_expand(h->cf, h->d_arena, h->d_tab_off, h->d_vm, parents, F, n_parent, children, rewards,
+    launch_expand(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, parents, F, n_parent, children, rewards,
                   done, hashes, as_stream(stream));
     return launch_check(h, "expand kernel");
 }

@@ -1,30 +1,35 @@
 // kernels.cuh -- device code of libautoverse.so (sm_103a).
 //
-// One CTA owns one environment (one board).  Each step:
-//   A. board + force tile -> bit-planes in shared memory: plane c is the
-//      board's channel-c bits as a row-major bit string of H*W bits, built
-//      32 cells at a time with one warp ballot per channel.  Every plane word
-//      j is stored doubled as (word j, word j+1) so that any 32-bit window of
-//      the bit string is one 64-bit shared load plus one funnel shift.
-//   B. matching (Sec. 2.1, ReLU(conv_{K_I}(D) - I + 1) == 1, evaluated as
-//      bitwise AND): a work item is (rule rotation, anchor word a); its 32
-//      bits are the anchors p = 32a + b.  Each term (channel c, window offset
-//      s = i*W + k, present/absent) ANDs in bit p+s of plane c (or its
-//      complement); the loop stops as soon as no anchor is left.  A match
-//      pays the rule's reward and ORs the rule's output (set | clear << 16)
-//      into a per-cell accumulator with shared-memory atomics: the
-//      transposed-convolution write of Sec. 2.1.
-//   C. combine next = (D & ~CLR) | (~D & SET) (force dropped), goal test by
-//      a block-wide OR, reward by warp reductions.
+// State representation.  A board lives on chip as bit-planes: plane c holds
+// channel c of every cell as a row-major bit string of H*W bits (cell p = y*W
+// + x is bit p & 31 of word p >> 5).  Plane C is the transient force channel.
+// Each plane word j is stored doubled as the pair (word j, word j+1), so any
+// 32-bit window of a bit string is one 64-bit shared load plus one funnel
+// shift.  A fused rollout keeps the planes resident for all its steps; cells
+// are touched only when boards enter or leave the kernel.
 //
-// Rule table layout (uint32 words, one table per env or one shared table):
-//   [0] K = 4R rule rotations   [1] n_items   [2] items_off   [3] terms_off
-//   [4] outs_off (even)          [5..7] 0
-//   [8 + 8*rr ...] header of rotation rr: shape = (h'-1)*5 + (w'-1),
-//        n_terms, n_outs, reward, first term, first out, 0, 0
-//   items:  (rr << 16) | a, every anchor word that holds a valid anchor
-//   terms:  (byte offset of plane c, word s>>5) << 8 | absent << 5 | (s & 31)
-//   outs:   pairs (cell offset i*W + k, set | clear << 16)
+// Matching (Sec. 2.1: a pattern matches where ReLU(conv_{K_I}(D) - I + 1) = 1,
+// i.e. every present entry is set and, with absent entries as -1 weights,
+// every absent entry is clear) is a bitwise AND over anchors: for anchor word
+// a (anchors p = 32a .. 32a+31) and a term (channel c, window offset
+// s = i*W + k), the anchors that pass are bits p + s of plane c.  One warp
+// takes one rule; its four quarter-warps take the rule's four rotations (a
+// rotation keeps the number of terms, so the quarters run the same loop), and
+// lane q of a quarter owns anchor words q, q+8, q+16, ...  Terms are ordered
+// so that the most selective come first; the warp leaves the rule as soon as
+// no lane has a live anchor.  A live match pays the rule's reward per anchor
+// and ORs the rule's output pattern into SET / CLEAR planes with shared
+// atomics (the transposed-convolution write of Sec. 2.1).  Then
+// next = (D & ~CLEAR) | (~D & SET), force dropped.
+//
+// Rule table layout (uint32 words; one table per env, or one shared):
+//   [0] R   [1] total terms   [2] total outputs   [3] 0
+//   [4 + 8r ...] rule r: n_present, n_absent, n_out, reward,
+//                        first term, first output, shapes (rotation g in byte g:
+//                        (h'-1)*5 + (w'-1)), 0
+//   terms   (uint2, 16-byte aligned, [term][rotation]):
+//           (byte offset of plane entry c*NWP + (s >> 5), s & 31)
+//   outputs (uint4, [output][rotation]): (s >> 5, s & 31, set bits, clear bits)
 #pragma once
 
 #include <cuda_runtime.h>
@@ -33,21 +38,28 @@
 namespace av {
 
 constexpr int kThreads = 256;
-constexpr int kPlanePad = 10;     // doubled-plane entries past the last word
-constexpr int kMaxCand = 4096;    // av_select: candidates per env
+constexpr int kWarps = kThreads / 32;
+constexpr int kPlanePad = 10;   // zero entries past the last anchor slot of a plane
+constexpr int kShapes = 25;     // (h', w') in 1..5 x 1..5
+constexpr int kMaxCand = 4096;  // av_select: candidates per env
+constexpr int kActChunk = 256;  // actions drawn ahead, per CTA
+constexpr int kMaxSmemRuleWords = 8192;  // stage a rule table in shared memory up to 32 KiB
 constexpr uint32_t kStatusVisitedOverflow = 1u;
 constexpr uint32_t kWarnAction = 1u;
 
 struct DevConfig {
-    int B, H, W, C, HW, NW, NWP, pstride;
+    int B, H, W, C, HW, NW, NWP, NA;  // NW plane words; NWP doubled entries per plane; NA words per lane
     int R, rules_per_env, max_steps, auto_reset;
     int ch_player, ch_goal, ch_empty, ch_wall, border_wall, cum_per_env;
     int cell_bytes;
+    int rule_words;  // largest rule table (words) when tables are staged in shared memory, else 0
 };
 
-__host__ __device__ inline uint32_t encode_term(int c, int s, int neg, int pstride)
+// Rule-table helpers shared by host (compiler) and device (reader).
+__host__ __device__ inline uint32_t table_terms_word(int R) { return 4u + 8u * (uint32_t)R; }
+__host__ __device__ inline uint32_t table_outs_word(int R, uint32_t total_terms)
 {
-    return ((uint32_t)(c * pstride + (s >> 5) * 8) << 8) | ((uint32_t)neg << 5) | (uint32_t)(s & 31);
+    return table_terms_word(R) + 8u * total_terms;  // 4 rotations x uint2 per term
 }
 
 // ------------------------------------------------------------------ RNG
@@ -76,263 +88,461 @@ __device__ __forceinline__ uint32_t uniform_below(uint64_t d, uint32_t n)
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 
 struct StepSmem {
-    size_t planes, sc, boards, red, total;
+    size_t planes, setp, clrp, basep, vm, masks, red, acts, rules, cells, total;
 };
 
-// Layout: planes | SC accumulators | n_boards boards of uint16 cells | 3 reward slots
-__host__ __device__ inline StepSmem step_smem(const DevConfig &cf, int n_boards)
+// planes | SET | CLEAR | base planes (initial map, or a child) | valid-anchor
+// masks [25][NW] | column masks [3][NW] | per-warp rewards + flags | cells
+__host__ __device__ inline StepSmem step_smem(const DevConfig &cf, int n_cell_boards)
 {
     StepSmem s;
+    const size_t pw = (size_t)cf.C * cf.NW * 4;
     s.planes = 0;
-    s.sc = align16((size_t)(cf.C + 1) * cf.NWP * 8);
-    s.boards = align16(s.sc + (size_t)cf.HW * 4);
-    s.red = align16(s.boards + (size_t)cf.HW * 2 * n_boards);
-    s.total = s.red + 16;
+    s.setp = align16((size_t)(cf.C + 1) * cf.NWP * 8);
+    s.clrp = align16(s.setp + pw);
+    s.basep = align16(s.clrp + pw);
+    s.vm = align16(s.basep + pw);
+    s.masks = align16(s.vm + (size_t)kShapes * cf.NW * 4);
+    s.red = align16(s.masks + (size_t)3 * cf.NW * 4);
+    s.acts = align16(s.red + (size_t)(kWarps + 4) * 4);
+    s.rules = align16(s.acts + kActChunk);
+    s.cells = align16(s.rules + (size_t)cf.rule_words * 4);
+    s.total = align16(s.cells + (size_t)n_cell_boards * cf.HW * 2);
     return s;
 }
 
-struct StepOut {
-    int reward;
-    int goal_left;
+struct Smem {
+    uint2 *planes;
+    uint32_t *setp, *clrp, *basep, *vm, *masks, *rules;
+    int *red, *flags;
+    uint8_t *acts;
+    uint16_t *cells;
 };
 
-// One transition of the board in `gin` into `gout` (both shared, uint16 cells).
-// `slot` is a zeroed shared int used for the block's reward sum.
-__device__ StepOut step_body(const DevConfig &cf, const uint32_t *__restrict__ tab,
-                             const uint32_t *__restrict__ vm, uint2 *planes, uint32_t *SC,
-                             const uint16_t *gin, uint16_t *gout, int action, int *slot)
+__device__ __forceinline__ Smem carve(unsigned char *smem, const DevConfig &cf, int n_cell_boards)
+{
+    const StepSmem L = step_smem(cf, n_cell_boards);
+    Smem m;
+    m.planes = reinterpret_cast<uint2 *>(smem + L.planes);
+    m.setp = reinterpret_cast<uint32_t *>(smem + L.setp);
+    m.clrp = reinterpret_cast<uint32_t *>(smem + L.clrp);
+    m.basep = reinterpret_cast<uint32_t *>(smem + L.basep);
+    m.vm = reinterpret_cast<uint32_t *>(smem + L.vm);
+    m.masks = reinterpret_cast<uint32_t *>(smem + L.masks);
+    m.red = reinterpret_cast<int *>(smem + L.red);
+    m.flags = m.red + kWarps;
+    m.acts = smem + L.acts;
+    m.rules = reinterpret_cast<uint32_t *>(smem + L.rules);
+    m.cells = reinterpret_cast<uint16_t *>(smem + L.cells);
+    return m;
+}
+
+// Zero planes and SET/CLEAR, stage the anchor and column masks.
+__device__ void stage_common(const DevConfig &cf, const Smem &S, const uint32_t *__restrict__ vm_g,
+                             const uint32_t *__restrict__ masks_g)
+{
+    const int tid = threadIdx.x;
+    for (int i = tid; i < (cf.C + 1) * cf.NWP; i += kThreads)
+        S.planes[i] = make_uint2(0u, 0u);
+    for (int i = tid; i < cf.C * cf.NW; i += kThreads) {
+        S.setp[i] = 0u;
+        S.clrp[i] = 0u;
+    }
+    for (int i = tid; i < kShapes * cf.NW; i += kThreads)
+        S.vm[i] = __ldg(vm_g + i);
+    for (int i = tid; i < 3 * cf.NW; i += kThreads)
+        S.masks[i] = __ldg(masks_g + i);
+    if (tid < kWarps + 4)
+        S.red[tid] = 0;
+}
+
+// Copy one env's rule table (n words, 16-byte aligned) into shared memory.
+__device__ void stage_rules(const uint32_t *__restrict__ tab, uint32_t n, uint32_t *dst)
+{
+    const uint4 *src = reinterpret_cast<const uint4 *>(tab);
+    uint4 *d = reinterpret_cast<uint4 *>(dst);
+    for (uint32_t i = threadIdx.x; i < n / 4; i += kThreads)
+        d[i] = __ldg(src + i);
+}
+
+template <bool SM>
+__device__ __forceinline__ uint4 ld4(const uint32_t *p)
+{
+    if (SM)
+        return *reinterpret_cast<const uint4 *>(p);
+    return __ldg(reinterpret_cast<const uint4 *>(p));
+}
+
+template <bool SM>
+__device__ __forceinline__ uint2 ld2(const uint2 *p)
+{
+    if (SM)
+        return *p;
+    return __ldg(p);
+}
+
+// Write plane word w of channel c into the doubled layout.
+__device__ __forceinline__ void put_word(uint2 *planes, int NWP, int c, int w, uint32_t v)
+{
+    planes[c * NWP + w].x = v;
+    if (w > 0)
+        planes[c * NWP + w - 1].y = v;
+}
+
+// Board cells (global) -> tile planes: one warp ballot per channel per 32 cells.
+// Writes the doubled planes when `dbl` is set, else plain words into `flat`.
+template <typename CellT>
+__device__ void cells_to_planes(const DevConfig &cf, const CellT *__restrict__ src, uint2 *dbl,
+                                uint32_t *flat)
 {
     const int tid = threadIdx.x, lane = tid & 31;
-    const int HW = cf.HW, H = cf.H, W = cf.W, C = cf.C, NCH = C + 1, NWP = cf.NWP;
-
-    // ---- A: board + force -> bit-planes
-    int dy = 0, dx = 0;
-    if (cf.ch_player >= 0) {
-        if (action == 1) dy = -1;
-        else if (action == 2) dx = 1;
-        else if (action == 3) dy = 1;
-        else if (action == 4) dx = -1;
-    }
-    const bool force = (dy | dx) != 0;
-    for (int base = 0; base < HW; base += blockDim.x) {
+    for (int base = 0; base < cf.HW; base += kThreads) {
         const int p = base + tid;
-        uint32_t v = 0;
-        if (p < HW) {
-            v = gin[p];
-            if (force) {
-                const int y = p / W, x = p - y * W;
-                const int sy = y - dy, sx = x - dx;
-                if ((unsigned)sy < (unsigned)H && (unsigned)sx < (unsigned)W &&
-                    ((gin[sy * W + sx] >> cf.ch_player) & 1u))
-                    v |= 1u << C;
-            }
-        }
-        const int w = p >> 5;
-        for (int c = 0; c < NCH; ++c) {
+        const uint32_t v = p < cf.HW ? (uint32_t)src[p] : 0u;
+        const int w = p >> 5;  // warp-uniform
+        for (int c = 0; c < cf.C; ++c) {
             const uint32_t bits = __ballot_sync(0xffffffffu, (v >> c) & 1u);
             if (lane == 0 && w < cf.NW) {
-                planes[c * NWP + w].x = bits;
-                if (w > 0)
-                    planes[c * NWP + w - 1].y = bits;
+                if (dbl)
+                    put_word(dbl, cf.NWP, c, w, bits);
+                else
+                    flat[c * cf.NW + w] = bits;
             }
         }
     }
-    __syncthreads();
+}
 
-    // ---- B: match every (rule rotation, anchor word) item
-    const uint32_t n_items = tab[1];
-    const uint32_t *items = tab + tab[2];
-    const uint32_t *terms = tab + tab[3];
-    const uint2 *outs = reinterpret_cast<const uint2 *>(tab + tab[4]);
-    const uint32_t *hdr = tab + 8;
-    const char *pbase = reinterpret_cast<const char *>(planes);
-    int rew = 0;
-    for (uint32_t it = tid; it < n_items; it += blockDim.x) {
-        const uint32_t item = __ldg(items + it);
-        const uint32_t rr = item >> 16, a = item & 0xffffu;
-        const uint4 h0 = __ldg(reinterpret_cast<const uint4 *>(hdr + 8 * rr));
-        const uint2 h1 = __ldg(reinterpret_cast<const uint2 *>(hdr + 8 * rr + 4));
-        uint32_t m = __ldg(vm + h0.x * cf.NW + a);
-        const char *abase = pbase + a * 8;
-        const uint32_t *tp = terms + h1.x;
-        for (uint32_t t = 0; t < h0.y && m; ++t) {
-            const uint32_t e = __ldg(tp + t);
-            const uint2 wd = *reinterpret_cast<const uint2 *>(abase + (e >> 8));
-            const uint32_t x = __funnelshift_r(wd.x, wd.y, e & 31u);
-            m &= (e & 32u) ? ~x : x;
-        }
-        if (m) {
-            rew += (int)h0.w * __popc(m);
-            const uint2 *op = outs + h1.y;
-            uint32_t mm = m;
-            while (mm) {
-                const int b = __ffs(mm) - 1;
-                mm &= mm - 1;
-                const int p = (int)a * 32 + b;
-                for (uint32_t o = 0; o < h0.z; ++o) {
-                    const uint2 ov = __ldg(op + o);
-                    atomicOr(&SC[p + (int)ov.x], ov.y);
+// Cell p of a plane set (doubled or flat).
+__device__ __forceinline__ uint32_t gather_cell(const DevConfig &cf, const uint2 *dbl,
+                                                const uint32_t *flat, int p)
+{
+    const int w = p >> 5, b = p & 31;
+    uint32_t v = 0;
+    for (int c = 0; c < cf.C; ++c) {
+        const uint32_t word = dbl ? dbl[c * cf.NWP + w].x : flat[c * cf.NW + w];
+        v |= ((word >> b) & 1u) << c;
+    }
+    return v;
+}
+
+// Force plane for `action`, from the player plane (warp-cooperative, one warp).
+// Player at p puts force at p + d: d = -W up, +1 right, +W down, -1 left,
+// dropped where it would leave the board.
+__device__ void write_force(const DevConfig &cf, const Smem &S, int action)
+{
+    const int lane = threadIdx.x & 31, NW = cf.NW, NWP = cf.NWP;
+    const uint32_t *firstcol = S.masks, *lastcol = S.masks + NW, *cellmask = S.masks + 2 * NW;
+    const bool on = cf.ch_player >= 0 && action >= 1 && action <= 4;
+    const uint2 *P = S.planes + (on ? cf.ch_player : 0) * NWP;
+    for (int w = lane; w < NW; w += 32) {
+        uint32_t f = 0;
+        if (on) {
+            const int n = (action == 1 || action == 3) ? cf.W : 1;
+            const int q = n >> 5, r = n & 31;
+            if (action == 1 || action == 4) {  // toward lower p: bits [32w + n, 32w + n + 32)
+                const uint2 e = P[w + q];
+                f = __funnelshift_r(e.x, e.y, r);
+            } else {  // toward higher p: bits [32w - n, 32w - n + 32)
+                const int j = w - q;
+                if (j >= 1) {
+                    const uint2 e = P[j - 1];
+                    f = __funnelshift_l(e.x, e.y, r);
+                } else if (j == 0) {
+                    f = P[0].x << r;
                 }
             }
+            if (action == 2)
+                f &= ~firstcol[w];
+            else if (action == 4)
+                f &= ~lastcol[w];
+            f &= cellmask[w];
+        }
+        put_word(S.planes, NWP, cf.C, w, f);
+    }
+}
+
+__device__ __forceinline__ void scatter_bits(uint32_t *dst, uint32_t chans, int NW, int w0, uint32_t lo,
+                                             uint32_t hi)
+{
+    while (chans) {
+        const int c = __ffs(chans) - 1;
+        chans &= chans - 1;
+        if (lo)
+            atomicOr(&dst[c * NW + w0], lo);
+        if (hi)
+            atomicOr(&dst[c * NW + w0 + 1], hi);
+    }
+}
+
+// One warp evaluates rule r in its four rotations over every anchor; returns
+// this lane's share of the reward and ORs the outputs of live matches into
+// the SET / CLEAR planes.  Present terms AND in the window bits, absent terms
+// AND in their complement; two terms per warp vote, and the warp leaves as
+// soon as no lane has a live anchor.
+template <int NA, bool SM>
+__device__ __forceinline__ int match_rule(const DevConfig &cf, const uint32_t *tab, int r, const Smem &S)
+{
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);  // n_present, n_absent, n_out, reward
+    const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);  // first term, first output, shapes
+    const int shape = (int)((h1.z >> (8 * g)) & 0xffu);
+    const uint32_t *vmr = S.vm + shape * cf.NW;
+    uint32_t m[NA];
+#pragma unroll
+    for (int u = 0; u < NA; ++u) {
+        const int a = q + 8 * u;
+        m[u] = a < cf.NW ? vmr[a] : 0u;
+    }
+    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)h1.x * 4 + g;
+    const unsigned char *pb = reinterpret_cast<const unsigned char *>(S.planes) + q * 8;
+    const uint32_t np = h0.x, nt = h0.x + h0.y;
+    uint32_t t = 0;
+    for (; t < nt; t += 2) {
+        const bool two = t + 1 < nt && (t + 1 < np || t >= np);
+        const uint32_t neg = t < np ? 0u : 0xffffffffu;
+        const uint2 d0 = ld2<SM>(tp + 4 * t);
+        const uint2 d1 = two ? ld2<SM>(tp + 4 * t + 4) : d0;
+        uint32_t any = 0;
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            const uint2 w0 = *reinterpret_cast<const uint2 *>(pb + d0.x + 64 * u);
+            const uint2 w1 = *reinterpret_cast<const uint2 *>(pb + d1.x + 64 * u);
+            const uint32_t x0 = __funnelshift_r(w0.x, w0.y, d0.y) ^ neg;
+            const uint32_t x1 = __funnelshift_r(w1.x, w1.y, d1.y) ^ neg;
+            m[u] &= x0 & x1;
+            any |= m[u];
+        }
+        if (!two)
+            t -= 1;  // consumed one term
+        if (!__any_sync(0xffffffffu, any != 0u))
+            return 0;
+    }
+    uint32_t cnt = 0;
+#pragma unroll
+    for (int u = 0; u < NA; ++u)
+        cnt += __popc(m[u]);
+    if (cnt == 0)
+        return 0;
+    const uint4 *op = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, tab[1])) + (size_t)h1.y * 4 + g;
+    for (uint32_t o = 0; o < h0.z; ++o) {
+        const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            if (!m[u])
+                continue;
+            const int w0 = q + 8 * u + (int)ov.x;
+            const uint32_t lo = m[u] << ov.y;
+            const uint32_t hi = ov.y ? (m[u] >> (32u - ov.y)) : 0u;
+            scatter_bits(S.setp, ov.z, cf.NW, w0, lo, hi);
+            scatter_bits(S.clrp, ov.w, cf.NW, w0, lo, hi);
         }
     }
-    rew = __reduce_add_sync(0xffffffffu, rew);
-    if (lane == 0 && rew)
-        atomicAdd(slot, rew);
-    __syncthreads();
+    S.flags[0] = 1;
+    return (int)h0.w * (int)cnt;
+}
 
-    // ---- C: combine, goal test
-    const uint32_t tiles = (1u << C) - 1u;
-    int any_goal = 0;
-    for (int p = tid; p < HW; p += blockDim.x) {
-        const uint32_t v = gin[p];
-        const uint32_t sc = SC[p];
-        if (sc)
-            SC[p] = 0;
-        const uint32_t set = sc & 0xffffu, clr = sc >> 16;
-        const uint32_t nv = ((v & ~clr) | (~v & set)) & tiles;
-        gout[p] = (uint16_t)nv;
-        if (cf.ch_goal >= 0)
-            any_goal |= (int)((nv >> cf.ch_goal) & 1u);
+// All warps: every rule; per-warp reward sums land in S.red[warp].
+template <int NA, bool SM>
+__device__ __forceinline__ void match_all(const DevConfig &cf, const uint32_t *tab, const Smem &S)
+{
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int rew = 0;
+    for (int r = warp; r < cf.R; r += kWarps)
+        rew += match_rule<NA, SM>(cf, tab, r, S);
+    rew = __reduce_add_sync(0xffffffffu, rew);
+    if (lane == 0)
+        S.red[warp] = rew;
+}
+
+__device__ __forceinline__ int action_at(const uint8_t *__restrict__ actions, uint64_t seed, int env, int s,
+                                         int *warn_flag)
+{
+    int a = actions ? (int)actions[env] : (int)uniform_below(draw(seed, 4, (uint64_t)env, 0, (uint64_t)s), 5);
+    if (a > 4) {
+        *warn_flag = 1;
+        a = 0;
     }
-    StepOut o;
-    o.goal_left = __syncthreads_or(any_goal);
-    if (cf.ch_goal < 0)
-        o.goal_left = 1;
-    o.reward = *slot;
-    return o;
+    return a;
+}
+
+// Actions of steps [s0, s0 + kActChunk) into the ring S.acts (one per thread).
+__device__ __forceinline__ void fill_actions(const uint8_t *__restrict__ actions, uint64_t seed, int env, int s0,
+                                             int n_steps, const Smem &S)
+{
+    const int s = s0 + (int)threadIdx.x;
+    if (threadIdx.x < kActChunk && s < n_steps)
+        S.acts[s & (kActChunk - 1)] = (uint8_t)action_at(actions, seed, env, s, S.flags + 1);
 }
 
 // ---------------------------------------------------------------- kernels
-template <typename CellT>
+// Fused rollout (n_steps >= 1).  With `actions` non-null the action of step
+// s is actions[env] (used by av_step, n_steps = 1); else it is drawn.
+// SM: the env's rule table is staged in shared memory.
+template <typename CellT, int NA, bool SM>
 __global__ void __launch_bounds__(kThreads)
 rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
-               const uint32_t *__restrict__ vm, CellT *cur, const CellT *__restrict__ init,
-               int32_t *tsteps, int n_steps, uint64_t seed, const uint8_t *__restrict__ actions,
-               CellT *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
-               uint32_t *status)
+               const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
+               const CellT *__restrict__ init, int32_t *tsteps, int n_steps, uint64_t seed,
+               const uint8_t *__restrict__ actions, CellT *obs_traj, int32_t *rew_traj,
+               uint8_t *done_traj, int32_t *rew_sum, uint32_t *status)
 {
     extern __shared__ __align__(16) unsigned char smem[];
-    const StepSmem L = step_smem(cf, 3);
-    const int env = blockIdx.x, tid = threadIdx.x, HW = cf.HW;
-    uint2 *planes = reinterpret_cast<uint2 *>(smem + L.planes);
-    uint32_t *SC = reinterpret_cast<uint32_t *>(smem + L.sc);
-    uint16_t *G0 = reinterpret_cast<uint16_t *>(smem + L.boards);
-    uint16_t *G1 = G0 + HW, *GI = G1 + HW;
-    int *red = reinterpret_cast<int *>(smem + L.red);
-    const uint32_t *tab = arena + tab_off[cf.rules_per_env ? env : 0];
+    const Smem S = carve(smem, cf, 0);
+    const int env = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int HW = cf.HW, NW = cf.NW, NWP = cf.NWP, C = cf.C;
+    const int table = cf.rules_per_env ? env : 0;
+    const uint32_t *tab_g = arena + tab_off[table];
+    const uint32_t *tab = SM ? S.rules : tab_g;
 
-    for (int i = tid; i < (cf.C + 1) * cf.NWP; i += blockDim.x)
-        planes[i] = make_uint2(0u, 0u);
-    const CellT *src = cur + (size_t)env * HW;
-    const CellT *isrc = init + (size_t)env * HW;
-    for (int p = tid; p < HW; p += blockDim.x) {
-        SC[p] = 0;
-        G0[p] = (uint16_t)src[p];
-        GI[p] = (uint16_t)isrc[p];
-    }
-    if (tid < 3)
-        red[tid] = 0;
+    stage_common(cf, S, vm_g, masks_g);
+    if (SM)
+        stage_rules(tab_g, tab_off[table + 1] - tab_off[table], S.rules);
+    __syncthreads();
+    cells_to_planes<CellT>(cf, cur + (size_t)env * HW, S.planes, nullptr);
+    cells_to_planes<CellT>(cf, init + (size_t)env * HW, nullptr, S.basep);
+    fill_actions(actions, seed, env, 0, n_steps, S);
     __syncthreads();
 
     int t = tsteps[env];
     int sum = 0;
-    uint32_t warn = 0;
-    uint16_t *gin = G0, *gout = G1;
+    if (warp == 0)
+        write_force(cf, S, S.acts[0]);
+    __syncthreads();
+
     for (int s = 0; s < n_steps; ++s) {
-        int a = actions ? (int)actions[env] : (int)uniform_below(draw(seed, 4, (uint64_t)env, 0, (uint64_t)s), 5);
-        if (a > 4) {
-            warn = kWarnAction;
-            a = 0;
+        if (((s + 1) & (kActChunk - 1)) == 0)
+            fill_actions(actions, seed, env, s + 1, n_steps, S);
+        match_all<NA, SM>(cf, tab, S);
+        __syncthreads();
+        if (warp == 0) {
+            // combine: a bit changes where any match asks for it
+            if (S.flags[0]) {
+                for (int c = 0; c < C; ++c)
+                    for (int w = lane; w < NW; w += 32) {
+                        const int i = c * NW + w;
+                        const uint32_t d = S.planes[c * NWP + w].x, st = S.setp[i], cl = S.clrp[i];
+                        S.setp[i] = 0u;
+                        S.clrp[i] = 0u;
+                        put_word(S.planes, NWP, c, w, (d & ~cl) | (~d & st));
+                    }
+                __syncwarp();
+                if (lane == 0)
+                    S.flags[0] = 0;
+            }
+            int goal = cf.ch_goal < 0;
+            if (cf.ch_goal >= 0)
+                for (int w = lane; w < NW; w += 32)
+                    goal |= S.planes[cf.ch_goal * NWP + w].x != 0u;
+            goal = __any_sync(0xffffffffu, goal);
+            t += 1;
+            const int done = !goal || (cf.max_steps > 0 && t >= cf.max_steps);
+            if (done && cf.auto_reset) {
+                for (int c = 0; c < C; ++c)
+                    for (int w = lane; w < NW; w += 32)
+                        put_word(S.planes, NWP, c, w, S.basep[c * NW + w]);
+                t = 0;
+            }
+            int rew = lane < kWarps ? S.red[lane] : 0;
+            rew = __reduce_add_sync(0xffffffffu, rew);
+            sum += rew;
+            if (lane == 0) {
+                if (rew_traj)
+                    rew_traj[(size_t)s * cf.B + env] = rew;
+                if (done_traj)
+                    done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
+            }
+            __syncwarp();
+            if (s + 1 < n_steps)
+                write_force(cf, S, S.acts[(s + 1) & (kActChunk - 1)]);
         }
-        if (tid == 0)
-            red[(s + 1) % 3] = 0;
-        const StepOut o = step_body(cf, tab, vm, planes, SC, gin, gout, a, &red[s % 3]);
-        t += 1;
-        const int done = !o.goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
-        if (done && cf.auto_reset) {
-            for (int p = tid; p < HW; p += blockDim.x)
-                gout[p] = GI[p];
-            t = 0;
-            __syncthreads();
-        }
+        __syncthreads();
         if (obs_traj) {
             CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
-            for (int p = tid; p < HW; p += blockDim.x)
-                dst[p] = (CellT)gout[p];
+            for (int p = tid; p < HW; p += kThreads)
+                dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
         }
-        if (tid == 0) {
-            if (rew_traj)
-                rew_traj[(size_t)s * cf.B + env] = o.reward;
-            if (done_traj)
-                done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
-        }
-        sum += o.reward;
-        uint16_t *tmp = gin;
-        gin = gout;
-        gout = tmp;
     }
     CellT *dst = cur + (size_t)env * HW;
-    for (int p = tid; p < HW; p += blockDim.x)
-        dst[p] = (CellT)gin[p];
+    for (int p = tid; p < HW; p += kThreads)
+        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
     if (tid == 0) {
         tsteps[env] = t;
         if (rew_sum)
             rew_sum[env] = sum;
-        if (warn)
-            atomicOr(status + 1, warn);
+        if (S.flags[1])
+            atomicOr(status + 1, kWarnAction);
     }
 }
 
-template <typename CellT>
+// Tree-search expansion: one CTA per parent, the 5 children in turn.
+template <typename CellT, int NA, bool SM>
 __global__ void __launch_bounds__(kThreads)
 expand_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
-              const uint32_t *__restrict__ vm, const CellT *__restrict__ parents, int F,
-              const int32_t *__restrict__ n_parent, CellT *children, int32_t *rewards,
-              uint8_t *done, uint64_t *hashes)
+              const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g,
+              const CellT *__restrict__ parents, int F, const int32_t *__restrict__ n_parent,
+              CellT *children, int32_t *rewards, uint8_t *done, uint64_t *hashes)
 {
     extern __shared__ __align__(16) unsigned char smem[];
-    const StepSmem L = step_smem(cf, 6);
-    const int node = blockIdx.x, env = node / F, tid = threadIdx.x, HW = cf.HW;
+    const Smem S = carve(smem, cf, 5);
+    const int node = blockIdx.x, env = node / F, tid = threadIdx.x, warp = tid >> 5;
+    const int HW = cf.HW, NW = cf.NW, NWP = cf.NWP, C = cf.C;
     if (n_parent && node - env * F >= n_parent[env])
         return;  // block-uniform: an empty frontier slot
-    uint2 *planes = reinterpret_cast<uint2 *>(smem + L.planes);
-    uint32_t *SC = reinterpret_cast<uint32_t *>(smem + L.sc);
-    uint16_t *G0 = reinterpret_cast<uint16_t *>(smem + L.boards);
-    int *red = reinterpret_cast<int *>(smem + L.red);
-    const uint32_t *tab = arena + tab_off[cf.rules_per_env ? env : 0];
+    const int table = cf.rules_per_env ? env : 0;
+    const uint32_t *tab_g = arena + tab_off[table];
+    const uint32_t *tab = SM ? S.rules : tab_g;
 
-    for (int i = tid; i < (cf.C + 1) * cf.NWP; i += blockDim.x)
-        planes[i] = make_uint2(0u, 0u);
-    const CellT *src = parents + (size_t)node * HW;
-    for (int p = tid; p < HW; p += blockDim.x) {
-        SC[p] = 0;
-        G0[p] = (uint16_t)src[p];
-    }
-    if (tid < 3)
-        red[tid] = 0;
+    stage_common(cf, S, vm_g, masks_g);
+    if (SM)
+        stage_rules(tab_g, tab_off[table + 1] - tab_off[table], S.rules);
+    __syncthreads();
+    cells_to_planes<CellT>(cf, parents + (size_t)node * HW, S.planes, nullptr);
     __syncthreads();
 
     for (int a = 0; a < 5; ++a) {
-        uint16_t *gc = G0 + (size_t)(a + 1) * HW;
-        if (tid == 0)
-            red[(a + 1) % 3] = 0;
-        const StepOut o = step_body(cf, tab, vm, planes, SC, G0, gc, a, &red[a % 3]);
-        const size_t slot = (size_t)node * 5 + a;
-        CellT *dst = children + slot * HW;
-        for (int p = tid; p < HW; p += blockDim.x)
-            dst[p] = (CellT)gc[p];
+        if (warp == 0)
+            write_force(cf, S, a);
+        __syncthreads();
+        match_all<NA, SM>(cf, tab, S);
+        __syncthreads();
+        const int any = S.flags[0];
+        for (int i = tid; i < C * NW; i += kThreads) {  // child planes
+            const int c = i / NW, w = i - c * NW;
+            const uint32_t d = S.planes[c * NWP + w].x;
+            uint32_t v = d;
+            if (any) {
+                v = (d & ~S.clrp[i]) | (~d & S.setp[i]);
+                S.setp[i] = 0u;
+                S.clrp[i] = 0u;
+            }
+            S.basep[i] = v;
+        }
+        __syncthreads();
+        uint16_t *cells = S.cells + (size_t)a * HW;
+        CellT *dst = children + ((size_t)node * 5 + a) * HW;
+        int goal = 0;
+        for (int p = tid; p < HW; p += kThreads) {
+            const uint32_t v = gather_cell(cf, nullptr, S.basep, p);
+            cells[p] = (uint16_t)v;
+            dst[p] = (CellT)v;
+            if (cf.ch_goal >= 0)
+                goal |= (int)((v >> cf.ch_goal) & 1u);
+        }
+        const int goal_left = __syncthreads_or(goal) || cf.ch_goal < 0;
         if (tid == 0) {
-            rewards[slot] = o.reward;
+            int rew = 0;
+            for (int w = 0; w < kWarps; ++w)
+                rew += S.red[w];
+            rewards[(size_t)node * 5 + a] = rew;
             if (done)
-                done[slot] = (uint8_t)!o.goal_left;
+                done[(size_t)node * 5 + a] = (uint8_t)!goal_left;
+            S.flags[0] = 0;
         }
     }
-    // children are complete: every step ended with a block-wide barrier.
-    // FNV-1a 64 over the canonical bytes, one thread per child.
-    if ((tid & 31) == 0 && (tid >> 5) < 5) {
-        const int a = tid >> 5;
-        const uint16_t *gc = G0 + (size_t)(a + 1) * HW;
+    __syncthreads();
+    // FNV-1a 64 over the canonical bytes, one thread per child
+    if ((tid & 31) == 0 && warp < 5) {
+        const uint16_t *gc = S.cells + (size_t)warp * HW;
         uint64_t hsh = 0xcbf29ce484222325ULL;
         for (int p = 0; p < HW; ++p) {
             const uint32_t v = gc[p];
@@ -340,7 +550,7 @@ expand_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *
             if (sizeof(CellT) == 2)
                 hsh = (hsh ^ (v >> 8)) * 0x100000001b3ULL;
         }
-        hashes[(size_t)node * 5 + a] = hsh;
+        hashes[(size_t)node * 5 + warp] = hsh;
     }
 }
 
@@ -653,61 +863,107 @@ inline size_t select_smem_bytes(int F)
     return (size_t)n2 * sizeof(Key128) * 2 + (size_t)n2 * 8 + 64;
 }
 
+// Anchor words per lane: the smallest power of two with 8 * NA >= NW.
+inline int anchor_slots(int NW)
+{
+    int na = 1;
+    while (8 * na < NW)
+        na <<= 1;
+    return na;
+}
+
+#define AV_FOR_NA(MACRO, CELL) MACRO(CELL, 1) MACRO(CELL, 2) MACRO(CELL, 4) MACRO(CELL, 8) MACRO(CELL, 16)
+
 inline cudaError_t configure_kernels(const DevConfig &cf)
 {
+    (void)cf;
     const int big = 200 * 1024;
     cudaError_t e = cudaSuccess;
     auto set = [&](const void *fn) {
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, big);
     };
-    if (cf.cell_bytes == 1) {
-        set((const void *)rollout_kernel<uint8_t>);
-        set((const void *)expand_kernel<uint8_t>);
-        set((const void *)reset_kernel<uint8_t>);
-        set((const void *)select_kernel<uint8_t>);
-        set((const void *)search_init_kernel<uint8_t>);
-    } else {
-        set((const void *)rollout_kernel<uint16_t>);
-        set((const void *)expand_kernel<uint16_t>);
-        set((const void *)reset_kernel<uint16_t>);
-        set((const void *)select_kernel<uint16_t>);
-        set((const void *)search_init_kernel<uint16_t>);
-    }
+#define AV_SET(CELL, NA)                                       \
+    set((const void *)rollout_kernel<CELL, NA, true>);         \
+    set((const void *)rollout_kernel<CELL, NA, false>);        \
+    set((const void *)expand_kernel<CELL, NA, true>);          \
+    set((const void *)expand_kernel<CELL, NA, false>);
+    AV_FOR_NA(AV_SET, uint8_t)
+    AV_FOR_NA(AV_SET, uint16_t)
+#undef AV_SET
+    set((const void *)reset_kernel<uint8_t>);
+    set((const void *)reset_kernel<uint16_t>);
+    set((const void *)select_kernel<uint8_t>);
+    set((const void *)select_kernel<uint16_t>);
     return e;
 }
 
-inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
-                           const uint32_t *vm, void *cur, const void *init, int32_t *t, int n_steps,
-                           uint64_t seed, const uint8_t *actions, void *obs_traj, int32_t *rew_traj,
-                           uint8_t *done_traj, int32_t *rew_sum, uint32_t *status, cudaStream_t st)
+template <typename CellT, int NA>
+void rollout_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+               const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
+               const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj,
+               int32_t *rew_sum, uint32_t *status, cudaStream_t st)
 {
-    const size_t sm = step_smem(cf, 3).total;
-    if (cf.cell_bytes == 1)
-        rollout_kernel<uint8_t><<<cf.B, kThreads, sm, st>>>(
-            cf, arena, tab_off, vm, (uint8_t *)cur, (const uint8_t *)init, t, n_steps, seed, actions,
-            (uint8_t *)obs_traj, rew_traj, done_traj, rew_sum, status);
+    if (cf.rule_words > 0)
+        rollout_kernel<CellT, NA, true><<<cf.B, kThreads, step_smem(cf, 0).total, st>>>(
+            cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
+            (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
     else
-        rollout_kernel<uint16_t><<<cf.B, kThreads, sm, st>>>(
-            cf, arena, tab_off, vm, (uint16_t *)cur, (const uint16_t *)init, t, n_steps, seed, actions,
-            (uint16_t *)obs_traj, rew_traj, done_traj, rew_sum, status);
+        rollout_kernel<CellT, NA, false><<<cf.B, kThreads, step_smem(cf, 0).total, st>>>(
+            cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
+            (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
+}
+
+inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
+                           const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
+                           int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
+                           int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                           cudaStream_t st)
+{
+#define AV_CASE(CELL, NA)                                                                              \
+    case NA:                                                                                          \
+        rollout_t<CELL, NA>(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions,      \
+                            obs_traj, rew_traj, done_traj, rew_sum, status, st);                      \
+        break;
+    if (cf.cell_bytes == 1) {
+        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint8_t) }
+    } else {
+        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint16_t) }
+    }
+#undef AV_CASE
+}
+
+template <typename CellT, int NA>
+void expand_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+              const uint32_t *masks, const void *parents, int F, const int32_t *n_parent, void *children,
+              int32_t *rewards, uint8_t *done, uint64_t *hashes, cudaStream_t st)
+{
+    if (cf.rule_words > 0)
+        expand_kernel<CellT, NA, true><<<(unsigned)(cf.B * F), kThreads, step_smem(cf, 5).total, st>>>(
+            cf, arena, tab_off, vm, masks, (const CellT *)parents, F, n_parent, (CellT *)children, rewards,
+            done, hashes);
+    else
+        expand_kernel<CellT, NA, false><<<(unsigned)(cf.B * F), kThreads, step_smem(cf, 5).total, st>>>(
+            cf, arena, tab_off, vm, masks, (const CellT *)parents, F, n_parent, (CellT *)children, rewards,
+            done, hashes);
 }
 
 inline void launch_expand(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
-                          const uint32_t *vm, const void *parents, int F, const int32_t *n_parent,
-                          void *children, int32_t *rewards, uint8_t *done, uint64_t *hashes,
-                          cudaStream_t st)
+                          const uint32_t *vm, const uint32_t *masks, const void *parents, int F,
+                          const int32_t *n_parent, void *children, int32_t *rewards, uint8_t *done,
+                          uint64_t *hashes, cudaStream_t st)
 {
-    const size_t sm = step_smem(cf, 6).total;
-    const unsigned grid = (unsigned)(cf.B * F);
-    if (cf.cell_bytes == 1)
-        expand_kernel<uint8_t><<<grid, kThreads, sm, st>>>(cf, arena, tab_off, vm, (const uint8_t *)parents,
-                                                          F, n_parent, (uint8_t *)children, rewards, done,
-                                                          hashes);
-    else
-        expand_kernel<uint16_t><<<grid, kThreads, sm, st>>>(cf, arena, tab_off, vm, (const uint16_t *)parents,
-                                                           F, n_parent, (uint16_t *)children, rewards, done,
-                                                           hashes);
+#define AV_CASE(CELL, NA)                                                                              \
+    case NA:                                                                                          \
+        expand_t<CELL, NA>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards,    \
+                           done, hashes, st);                                                         \
+        break;
+    if (cf.cell_bytes == 1) {
+        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint8_t) }
+    } else {
+        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint16_t) }
+    }
+#undef AV_CASE
 }
 
 inline void launch_reset(const DevConfig &cf, const uint32_t *cum, uint64_t seed, void *cur, void *init,

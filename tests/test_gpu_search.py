@@ -100,17 +100,41 @@ def test_search_full_size_sampled():
     ids = sample_envs(wl.batch, 4, seed=4)
     ref = oracle.search(cfg, rules, to_np(roots)[ids], iters, k, env_ids=ids)
     _compare_search(gpu, ref, ids)
-    assert (to_np(gpu["trace_n"])[:, -1] > 0).any()
+    assert (to_np(gpu["trace_n"])[:, 0] > 0).any()
     env.sync()
+    env.close()
+
+
+def _maze(batch, capacity):
+    """The paper's base maze game (Sec. 2.2.1): move and eat rules, an open
+    16x16 board with border walls, one player and one food tile per env."""
+    from tests import golden_io
+    import paper_2407_04221_gb300 as av
+    fx = golden_io.load(golden_io.GOLDEN_DIR + "/03_eat_food.txt")
+    fields = dict(fx.cfg_fields(), batch=batch, H=16, W=16)
+    env = av.Env(fields, fx.rules, search_capacity=capacity)
+    g = np.full((batch, 16, 16), 1, np.uint8)  # floor
+    g[:, 0, :] = g[:, -1, :] = g[:, :, 0] = g[:, :, -1] = 2  # walls
+    for b in range(batch):
+        g[b, 2 + b % 5, 3] |= 4  # player
+        g[b, 11, 12 - b % 7] = 8  # food
+    return env, oracle.make_cfg(**fields), fx.rules, g
+
+
+def test_search_maze_reaches_food():
+    env, cfg, rules, g = _maze(7, 1 + 12 * 64)
+    roots = to_dev(g)
+    gpu = env.search(roots, 12, 64)
+    ref = oracle.search(cfg, rules, g, 12, 64)
+    _compare_search(gpu, ref, np.arange(7))
+    assert (ref["trace_best"].max(axis=1) == 1).any()  # some beam eats the food
     env.close()
 
 
 def test_visited_overflow_reports_device_error():
     import paper_2407_04221_gb300 as av
-    wl = wk.WORKLOADS[4].scaled(batch=2)
-    env, cfg, rules, cum = make(wl, 0, search_capacity=10)  # far too small for k=8 x 4
-    roots = env.reset(3)
-    env.search(roots, 4, 8)
+    env, cfg, rules, g = _maze(2, 10)  # far too small: 1 + 4 + 8 > 10 after two rounds
+    env.search(to_dev(g), 4, 8)
     with pytest.raises(av.AvError) as ei:
         env.sync()
     assert ei.value.status == av.AV_EDEVICE
