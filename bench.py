@@ -38,7 +38,11 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 KERNEL_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "kernels.cuh")
 PROFILE = os.path.join(ROOT, "profiles", "rollout_kernel_grid16_b1024.md")
 SM_COUNT_GB300 = 152
-INT_LANES_PER_SM = 64  # 32-bit integer logic/shift/add lanes per SM per clock (4 SMSPs x 16)
+# 32-bit integer instructions issued per SM per clock: 4 schedulers x 32 lanes.
+# The committed probe (--int-probe) reaches 113-114 of them for IADD3, SHF and
+# IMAD chains and 76 for LOP3 on GB300.
+INT_LANES_PER_SM = 128
+PROBE_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "probe", "int_issue_probe.cu")
 
 
 # ------------------------------------------------------------ workload
@@ -355,6 +359,17 @@ def run_ours(args, wl):
     return 0
 
 
+def run_int_probe() -> int:
+    """Build and run the integer-issue probe (needs nvcc and a GPU)."""
+    import tempfile
+    nvcc = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "bin", "nvcc")
+    with tempfile.TemporaryDirectory() as d:
+        exe = os.path.join(d, "int_issue_probe")
+        subprocess.check_call([nvcc if os.path.exists(nvcc) else "nvcc", "-O3", "-gencode",
+                               "arch=compute_103a,code=sm_103a", "-o", exe, PROBE_SRC])
+        return subprocess.call([exe])
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -364,7 +379,10 @@ def main(argv=None):
     ap.add_argument("--config", type=int, default=2, choices=(2, 3, 5))
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--int-probe", action="store_true", help="measure integer issue rate and exit")
     args = ap.parse_args(argv)
+    if args.int_probe:
+        return run_int_probe()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     wl = workload_for(args.config)
