@@ -184,6 +184,39 @@ int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *p
               int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live, int32_t *n_next,
               uintptr_t stream);
 
+/* Largest 2 * batch * capacity accepted by av_select_static (hashes). */
+#define AV_SELECT_STATIC_MAX_HASHES (1 << 21) /* 16 MiB of uint64 */
+
+/* av_select without a handle and without allocating anything.  For callers
+ * that cannot call cudaMalloc: code running under an allocator they do not
+ * own, inside a memory pool with a fixed budget, or in a process where a
+ * device allocation would break their own memory accounting.  The paper has
+ * no counterpart: this is a deployment variant of av_select.
+ *
+ * Same selection as av_select for boards of batch x H x W cells with C tile
+ * channels; the visited sets are caller-owned: visited uint64[batch][capacity]
+ * (device, env b's first n_visited[b] entries sorted ascending) and n_visited
+ * int32[batch] (device), both updated in place.  status: device uint32 or
+ * NULL; receives bit 0 when a visited set would exceed capacity (that env's
+ * set is then left unchanged).
+ *
+ * The working copy of the visited sets lives in one file-scope device array
+ * of AV_SELECT_STATIC_MAX_HASHES hashes that every GPU loading the library
+ * holds until the process exits; sizes with 2 * batch * capacity above it
+ * are rejected with AV_EINVAL before any GPU work.  The first call on a
+ * device looks up the array's device address (with that device current):
+ * make that first call before any stream capture.  All calls share the
+ * array, so calls that overlap on the GPU (other streams, other threads)
+ * race: serialise them.  No cudaMalloc, cudaFree or other allocation is
+ * made; the work is enqueued on `stream`. */
+int av_select_static(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t F,
+                     const int32_t *n_parent, const int32_t *parent_cum,
+                     const uint8_t *parent_live, const void *cand_grids,
+                     const int32_t *cand_reward, const uint8_t *cand_done,
+                     const uint64_t *cand_hash, int32_t k, void *next_grids, int32_t *next_cum,
+                     uint64_t *next_hash, uint8_t *next_live, int32_t *n_next, uint64_t *visited,
+                     int32_t *n_visited, int32_t capacity, uint32_t *status, uintptr_t stream);
+
 /* Wait for the handle's pending work (device-wide synchronise) and report
  * deferred errors: AV_ECUDA for a CUDA error, AV_EDEVICE when a kernel set
  * its error status (e.g. visited set overflow). */

@@ -22,8 +22,9 @@ AV_OK, AV_EINVAL, AV_ENOMEM, AV_ECUDA, AV_ESTATE, AV_EDEVICE = 0, -1, -2, -3, -4
 AV_WARN_ACTION = 1
 RULE_BYTES = 408
 EXPORTS = ("av_create", "av_destroy", "av_reset", "av_set_state", "av_get_state", "av_step",
-           "av_rollout", "av_expand", "av_search_init", "av_select", "av_sync", "av_warnings",
-           "av_strerror", "av_last_error")
+           "av_rollout", "av_expand", "av_search_init", "av_select", "av_select_static", "av_sync",
+           "av_warnings", "av_strerror", "av_last_error")
+AV_SELECT_STATIC_MAX_HASHES = 1 << 21
 
 
 class AvConfig(ctypes.Structure):
@@ -67,6 +68,8 @@ def load() -> ctypes.CDLL:
         "av_expand": [vp, vp, i32, vp, vp, vp, vp, vp, up],
         "av_search_init": [vp, vp, vp, vp, up],
         "av_select": [vp, i32, vp, vp, vp, vp, vp, vp, vp, i32, vp, vp, vp, vp, vp, up],
+        "av_select_static": [i32, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, i32, vp, vp, vp,
+                             vp, vp, vp, vp, i32, vp, up],
         "av_sync": [vp],
         "av_warnings": [vp, ctypes.POINTER(ctypes.c_uint32)],
     }
@@ -186,6 +189,22 @@ def av_select(h, F, n_parent, parent_cum, parent_live, cand_grids, cand_reward, 
                           int(k), _ptr(next_grids), _ptr(next_cum), _ptr(next_hash),
                           _ptr(next_live), _ptr(n_next), _stream(stream))
     _check(h, "av_select", rc)
+
+
+def av_select_static(batch, H, W, C, F, n_parent, parent_cum, parent_live, cand_grids,
+                     cand_reward, cand_done, cand_hash, k, next_grids, next_cum, next_hash,
+                     next_live, n_next, visited, n_visited, capacity, status=None, stream=None):
+    """av_select without a handle or any device allocation: the caller owns
+    the visited sets (visited [batch, capacity] uint64, n_visited [batch]);
+    the library's fixed working array holds the merge.  See the C header for
+    the size limit and for why overlapping calls must be serialised."""
+    rc = load().av_select_static(int(batch), int(H), int(W), int(C), int(F), _ptr(n_parent),
+                                 _ptr(parent_cum), _ptr(parent_live), _ptr(cand_grids),
+                                 _ptr(cand_reward), _ptr(cand_done), _ptr(cand_hash), int(k),
+                                 _ptr(next_grids), _ptr(next_cum), _ptr(next_hash), _ptr(next_live),
+                                 _ptr(n_next), _ptr(visited), _ptr(n_visited), int(capacity),
+                                 _ptr(status), _stream(stream))
+    _check(None, "av_select_static", rc)
 
 
 def av_sync(h):

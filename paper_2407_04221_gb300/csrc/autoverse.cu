@@ -552,6 +552,96 @@ int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *p
     return launch_check(h, "select kernel");
 }
 
+}  // extern "C"
+
+// ------------------------------------------------ av_select without allocation
+namespace {
+
+// Working copy of the visited sets for av_select_static: [2][batch][capacity]
+// (input copy, merged result) followed by a status word.  Lives as long as the
+// process, on every GPU that loads the library.
+constexpr size_t kStaticHashes = AV_SELECT_STATIC_MAX_HASHES;
+__device__ __align__(256) uint64_t g_select_scratch[kStaticHashes + 32];
+
+constexpr int kMaxDevices = 64;
+uint64_t *g_scratch_ptr[kMaxDevices] = {};  // device address of g_select_scratch, per device
+bool g_scratch_ready[kMaxDevices] = {};
+
+// Once per device, with it current: look up the array's device address (in
+// host code the symbol is only a stand-in) and allow select's shared memory.
+int static_scratch(uint64_t **out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return AV_ECUDA;
+    if (!g_scratch_ready[dev]) {
+        void *ptr = nullptr;
+        if (cudaGetSymbolAddress(&ptr, g_select_scratch) != cudaSuccess || !ptr)
+            return AV_ECUDA;
+        const int big = 200 * 1024;
+        if (cudaFuncSetAttribute((const void *)select_kernel<uint8_t>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, big) != cudaSuccess ||
+            cudaFuncSetAttribute((const void *)select_kernel<uint16_t>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, big) != cudaSuccess)
+            return AV_ECUDA;
+        g_scratch_ptr[dev] = static_cast<uint64_t *>(ptr);
+        g_scratch_ready[dev] = true;
+    }
+    *out = g_scratch_ptr[dev];
+    return AV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int av_select_static(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t F,
+                     const int32_t *n_parent, const int32_t *parent_cum,
+                     const uint8_t *parent_live, const void *cand_grids,
+                     const int32_t *cand_reward, const uint8_t *cand_done,
+                     const uint64_t *cand_hash, int32_t k, void *next_grids, int32_t *next_cum,
+                     uint64_t *next_hash, uint8_t *next_live, int32_t *n_next, uint64_t *visited,
+                     int32_t *n_visited, int32_t capacity, uint32_t *status, uintptr_t stream)
+{
+    if (batch < 1 || H < 1 || H > AV_MAX_SIDE || W < 1 || W > AV_MAX_SIDE || C < 1 || C > AV_MAX_C)
+        return AV_EINVAL;
+    if (F < 1 || 5 * F > kMaxCand || k < 1 || k > 5 * F || capacity < 1)
+        return AV_EINVAL;
+    if (2 * (size_t)batch * (size_t)capacity > kStaticHashes)
+        return AV_EINVAL;  // beyond the fixed working array
+    if (!n_parent || !parent_cum || !parent_live || !cand_grids || !cand_reward || !cand_done ||
+        !cand_hash || !next_grids || !next_cum || !next_hash || !next_live || !n_next || !visited ||
+        !n_visited)
+        return AV_EINVAL;
+    uint64_t *scratch = nullptr;
+    int rc = static_scratch(&scratch);
+    if (rc != AV_OK)
+        return rc;
+    DevConfig cf{};
+    cf.B = batch;
+    cf.H = H;
+    cf.W = W;
+    cf.C = C;
+    cf.HW = H * W;
+    cf.cell_bytes = C <= 8 ? 1 : 2;
+    cudaStream_t st = as_stream(stream);
+    const size_t n = (size_t)batch * capacity;
+    uint32_t *sstatus = reinterpret_cast<uint32_t *>(scratch + kStaticHashes);
+    if (cudaMemsetAsync(sstatus, 0, 4, st) != cudaSuccess ||
+        cudaMemcpyAsync(scratch, visited, n * 8, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+        return AV_ECUDA;
+    launch_select(cf, capacity, 0, F, n_parent, parent_cum, parent_live, cand_grids, cand_reward,
+                  cand_done, cand_hash, k, next_grids, next_cum, next_hash, next_live, n_next, scratch,
+                  n_visited, sstatus, st);
+    if (cudaGetLastError() != cudaSuccess)
+        return AV_ECUDA;
+    if (cudaMemcpyAsync(visited, scratch + n, n * 8, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+        return AV_ECUDA;
+    if (status && cudaMemcpyAsync(status, sstatus, 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+        return AV_ECUDA;
+    return AV_OK;
+}
+
 int av_sync(av_handle *h)
 {
     if (!h)
