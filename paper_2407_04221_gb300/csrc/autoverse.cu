@@ -20,7 +20,7 @@
 #include <string>
 #include <vector>
 
-#include "kernels.cuh"
+#include "launch.h"
 
 using namespace av;
 
@@ -145,10 +145,10 @@ void turn_position(int h, int w, int g, int &i, int &k)
 // Compile one rule table into the layout read by the kernels (kernels.cuh,
 // "Rule table layout").  The term order is chosen once on the base pattern
 // and carried through every rotation, so the four rotations of a rule run
-// the same loop: present entries first -- positions with more present
-// channels first (two present tile types at one cell rule each other out on
-// one-hot boards), then the force channel, the player channel, higher
-// channels -- and absent entries last.  Any order gives the same result.
+// the same loop: an exclusive pair of present tile channels first (see
+// below), then a present force term, positions with more present channels,
+// the player channel, higher channels; absent entries last.  Any order gives
+// the same result; a selective order lets evaluation stop early.
 void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32_t> &arena)
 {
     const size_t base = arena.size();
@@ -177,6 +177,25 @@ void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32
             if (a.key1 != b.key1) return a.key1 > b.key1;
             return a.c > b.c;
         });
+        // An exclusive pair leads when the rule has one: two present tile
+        // channels (neither the player's) at one position.  Initial maps hold
+        // one tile type per cell (the player overlays), so such a pair rules
+        // out every anchor at once until rules make cells multi-hot.
+        for (int i = 0, found = 0; i < p.h && !found; ++i)
+            for (int k = 0; k < p.w && !found; ++k) {
+                int picks[2], n = 0;
+                for (size_t u = 0; u < pres.size() && n < 2; ++u)
+                    if (pres[u].i == i && pres[u].k == k && pres[u].c < cf.C && pres[u].c != cf.ch_player)
+                        picks[n++] = (int)u;
+                if (n == 2) {
+                    const BT a = pres[picks[0]], b = pres[picks[1]];
+                    pres.erase(pres.begin() + picks[1]);
+                    pres.erase(pres.begin() + picks[0]);
+                    pres.insert(pres.begin(), b);
+                    pres.insert(pres.begin(), a);
+                    found = 1;
+                }
+            }
         uint32_t *hd = &hdr[8 * (size_t)r];
         hd[0] = (uint32_t)pres.size();
         hd[1] = (uint32_t)absn.size();
@@ -362,6 +381,14 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     cf.border_wall = cfg->border_wall ? 1 : 0;
     cf.cum_per_env = cfg->cum_per_env;
     cf.cell_bytes = cfg->C <= 8 ? 1 : 2;
+    // Kernel path override, for testing every path on the same shapes:
+    // AV_KERNEL_PATH=block forces the one-CTA-per-env kernels (default: the fast
+    // rollout and one-warp-per-parent expansion for boards of at most 16 plane
+    // words); AV_FAST_WARPS=8 runs the fast rollout with 8 warps per env.
+    if (const char *path = getenv("AV_KERNEL_PATH"))
+        cf.path = strcmp(path, "block") == 0 ? 1 : 0;
+    if (const char *fw = getenv("AV_FAST_WARPS"))
+        cf.fast_warps = atoi(fw) == 8 ? 8 : 4;
     h->grid_bytes = (size_t)cf.HW * cf.cell_bytes;
 
     std::vector<uint32_t> arena, tab_off((size_t)n_tables + 1);
@@ -421,7 +448,7 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
         delete h;
         return AV_ECUDA;
     }
-    if (configure_kernels(cf) != cudaSuccess) {
+    if (configure_kernels() != cudaSuccess) {
         free_all(h);
         delete h;
         return AV_ECUDA;
@@ -578,11 +605,7 @@ int static_scratch(uint64_t **out)
         void *ptr = nullptr;
         if (cudaGetSymbolAddress(&ptr, g_select_scratch) != cudaSuccess || !ptr)
             return AV_ECUDA;
-        const int big = 200 * 1024;
-        if (cudaFuncSetAttribute((const void *)select_kernel<uint8_t>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, big) != cudaSuccess ||
-            cudaFuncSetAttribute((const void *)select_kernel<uint16_t>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, big) != cudaSuccess)
+        if (configure_search() != cudaSuccess)
             return AV_ECUDA;
         g_scratch_ptr[dev] = static_cast<uint64_t *>(ptr);
         g_scratch_ready[dev] = true;

@@ -35,6 +35,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 namespace av {
 
 constexpr int kThreads = 256;
@@ -53,6 +55,8 @@ struct DevConfig {
     int ch_player, ch_goal, ch_empty, ch_wall, border_wall, cum_per_env;
     int cell_bytes;
     int rule_words;  // largest rule table (words) when tables are staged in shared memory, else 0
+    int path;        // 0: choose; 1: one CTA per env (block) kernels forced
+    int fast_warps;  // fast rollout: warps per environment (4, or 8 when set to 8)
 };
 
 // Rule-table helpers shared by host (compiler) and device (reader).
@@ -138,7 +142,7 @@ __device__ __forceinline__ Smem carve(unsigned char *smem, const DevConfig &cf, 
 }
 
 // Zero planes and SET/CLEAR, stage the anchor and column masks.
-__device__ void stage_common(const DevConfig &cf, const Smem &S, const uint32_t *__restrict__ vm_g,
+static __device__ void stage_common(const DevConfig &cf, const Smem &S, const uint32_t *__restrict__ vm_g,
                              const uint32_t *__restrict__ masks_g)
 {
     const int tid = threadIdx.x;
@@ -157,7 +161,7 @@ __device__ void stage_common(const DevConfig &cf, const Smem &S, const uint32_t 
 }
 
 // Copy one env's rule table (n words, 16-byte aligned) into shared memory.
-__device__ void stage_rules(const uint32_t *__restrict__ tab, uint32_t n, uint32_t *dst)
+static __device__ void stage_rules(const uint32_t *__restrict__ tab, uint32_t n, uint32_t *dst)
 {
     const uint4 *src = reinterpret_cast<const uint4 *>(tab);
     uint4 *d = reinterpret_cast<uint4 *>(dst);
@@ -228,12 +232,12 @@ __device__ __forceinline__ uint32_t gather_cell(const DevConfig &cf, const uint2
 // Force plane for `action`, from the player plane (warp-cooperative, one warp).
 // Player at p puts force at p + d: d = -W up, +1 right, +W down, -1 left,
 // dropped where it would leave the board.
-__device__ void write_force(const DevConfig &cf, const Smem &S, int action)
+static __device__ void force_plane(const DevConfig &cf, uint2 *planes, const uint32_t *masks, int action)
 {
     const int lane = threadIdx.x & 31, NW = cf.NW, NWP = cf.NWP;
-    const uint32_t *firstcol = S.masks, *lastcol = S.masks + NW, *cellmask = S.masks + 2 * NW;
+    const uint32_t *firstcol = masks, *lastcol = masks + NW, *cellmask = masks + 2 * NW;
     const bool on = cf.ch_player >= 0 && action >= 1 && action <= 4;
-    const uint2 *P = S.planes + (on ? cf.ch_player : 0) * NWP;
+    const uint2 *P = planes + (on ? cf.ch_player : 0) * NWP;
     for (int w = lane; w < NW; w += 32) {
         uint32_t f = 0;
         if (on) {
@@ -257,8 +261,13 @@ __device__ void write_force(const DevConfig &cf, const Smem &S, int action)
                 f &= ~lastcol[w];
             f &= cellmask[w];
         }
-        put_word(S.planes, NWP, cf.C, w, f);
+        put_word(planes, NWP, cf.C, w, f);
     }
+}
+
+__device__ __forceinline__ void write_force(const DevConfig &cf, const Smem &S, int action)
+{
+    force_plane(cf, S.planes, S.masks, action);
 }
 
 __device__ __forceinline__ void scatter_bits(uint32_t *dst, uint32_t chans, int NW, int w0, uint32_t lo,
@@ -554,6 +563,745 @@ expand_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *
     }
 }
 
+// ============================================================ warp-resident path
+// Small boards (at most 16 plane words): one warp owns one environment for a
+// whole launch, with its own planes, SET / CLEAR planes and staged rule table
+// in shared memory.  It evaluates the first two terms of RB rules together
+// (independent dependency chains), continues only the rules that still have a
+// live anchor, and then updates its board itself: no block-wide barrier.
+
+constexpr int kWarpCtaMax = 4;  // warps (= environments) per CTA at most
+
+struct WarpLayout {
+    size_t planes, setp, clrp, basep, vm, masks, acts, rules, cells, total;
+};
+
+__host__ __device__ inline WarpLayout warp_layout(const DevConfig &cf, int n_cell_boards)
+{
+    WarpLayout L;
+    const size_t pw = (size_t)cf.C * cf.NW * 4;
+    L.planes = 0;
+    L.setp = align16((size_t)(cf.C + 1) * cf.NWP * 8);
+    L.clrp = align16(L.setp + pw);
+    L.basep = align16(L.clrp + pw);
+    L.vm = align16(L.basep + pw);
+    L.masks = align16(L.vm + (size_t)kShapes * cf.NW * 4);
+    L.acts = align16(L.masks + (size_t)3 * cf.NW * 4);
+    L.rules = align16(L.acts + kActChunk);
+    L.cells = align16(L.rules + (size_t)cf.rule_words * 4);
+    L.total = align16(L.cells + (size_t)n_cell_boards * cf.HW * 2);
+    return L;
+}
+
+struct WarpSmem {
+    uint2 *planes;
+    uint32_t *setp, *clrp, *basep, *vm, *masks, *rules;
+    uint8_t *acts;
+    uint16_t *cells;
+};
+
+__device__ __forceinline__ WarpSmem carve_warp(unsigned char *smem, const DevConfig &cf, int n_cell_boards)
+{
+    const WarpLayout L = warp_layout(cf, n_cell_boards);
+    unsigned char *b = smem + (size_t)(threadIdx.x >> 5) * L.total;
+    WarpSmem m;
+    m.planes = reinterpret_cast<uint2 *>(b + L.planes);
+    m.setp = reinterpret_cast<uint32_t *>(b + L.setp);
+    m.clrp = reinterpret_cast<uint32_t *>(b + L.clrp);
+    m.basep = reinterpret_cast<uint32_t *>(b + L.basep);
+    m.vm = reinterpret_cast<uint32_t *>(b + L.vm);
+    m.masks = reinterpret_cast<uint32_t *>(b + L.masks);
+    m.acts = b + L.acts;
+    m.rules = reinterpret_cast<uint32_t *>(b + L.rules);
+    m.cells = reinterpret_cast<uint16_t *>(b + L.cells);
+    return m;
+}
+
+static __device__ void warp_stage(const DevConfig &cf, const WarpSmem &S, const uint32_t *__restrict__ vm_g,
+                           const uint32_t *__restrict__ masks_g, const uint32_t *__restrict__ tab_g,
+                           uint32_t tab_words, bool rules_to_smem)
+{
+    const int lane = threadIdx.x & 31;
+    for (int i = lane; i < (cf.C + 1) * cf.NWP; i += 32)
+        S.planes[i] = make_uint2(0u, 0u);
+    for (int i = lane; i < cf.C * cf.NW; i += 32) {
+        S.setp[i] = 0u;
+        S.clrp[i] = 0u;
+    }
+    for (int i = lane; i < kShapes * cf.NW; i += 32)
+        S.vm[i] = __ldg(vm_g + i);
+    for (int i = lane; i < 3 * cf.NW; i += 32)
+        S.masks[i] = __ldg(masks_g + i);
+    if (rules_to_smem) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(tab_g);
+        uint4 *d = reinterpret_cast<uint4 *>(S.rules);
+        for (uint32_t i = lane; i < tab_words / 4; i += 32)
+            d[i] = __ldg(src + i);
+    }
+    __syncwarp();
+}
+
+template <typename CellT>
+__device__ void warp_cells_to_planes(const DevConfig &cf, const CellT *__restrict__ src, uint2 *dbl,
+                                     uint32_t *flat)
+{
+    const int lane = threadIdx.x & 31;
+    for (int base = 0; base < cf.HW; base += 32) {
+        const int p = base + lane;
+        const uint32_t v = p < cf.HW ? (uint32_t)src[p] : 0u;
+        const int w = base >> 5;
+        for (int c = 0; c < cf.C; ++c) {
+            const uint32_t bits = __ballot_sync(0xffffffffu, (v >> c) & 1u);
+            if (lane == 0) {
+                if (dbl)
+                    put_word(dbl, cf.NWP, c, w, bits);
+                else
+                    flat[c * cf.NW + w] = bits;
+            }
+        }
+    }
+}
+
+template <int NA>
+struct Words {
+    uint32_t v[NA];
+};
+
+// Remaining terms of a rule that survived its first two, then its write.
+// Returns (this lane's reward, 1 if this lane wrote an output).
+template <int NA, bool SM>
+__device__ __noinline__ int2 warp_rule_rest(const DevConfig &cf, const uint32_t *tab, const WarpSmem &S, int r,
+                                            Words<NA> mw)
+{
+    uint32_t *m = mw.v;
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
+    const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
+    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)h1.x * 4 + g;
+    const unsigned char *pb = reinterpret_cast<const unsigned char *>(S.planes) + q * 8;
+    const uint32_t np = h0.x, nt = h0.x + h0.y;
+    for (uint32_t t = 2; t < nt; t += 2) {
+        const bool two = t + 1 < nt && (t + 1 < np || t >= np);
+        const uint32_t neg = t < np ? 0u : 0xffffffffu;
+        const uint2 d0 = ld2<SM>(tp + 4 * t);
+        const uint2 d1 = two ? ld2<SM>(tp + 4 * t + 4) : d0;
+        uint32_t any = 0;
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            const uint2 w0 = *reinterpret_cast<const uint2 *>(pb + d0.x + 64 * u);
+            const uint2 w1 = *reinterpret_cast<const uint2 *>(pb + d1.x + 64 * u);
+            m[u] &= (__funnelshift_r(w0.x, w0.y, d0.y) ^ neg) & (__funnelshift_r(w1.x, w1.y, d1.y) ^ neg);
+            any |= m[u];
+        }
+        if (!two)
+            t -= 1;
+        if (!__any_sync(0xffffffffu, any != 0u))
+            return make_int2(0, 0);
+    }
+    uint32_t cnt = 0;
+#pragma unroll
+    for (int u = 0; u < NA; ++u)
+        cnt += __popc(m[u]);
+    if (cnt == 0)
+        return make_int2(0, 0);
+    const uint4 *op = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, tab[1])) + (size_t)h1.y * 4 + g;
+    for (uint32_t o = 0; o < h0.z; ++o) {
+        const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            if (!m[u])
+                continue;
+            const int w0 = q + 8 * u + (int)ov.x;
+            const uint32_t lo = m[u] << ov.y;
+            const uint32_t hi = ov.y ? (m[u] >> (32u - ov.y)) : 0u;
+            scatter_bits(S.setp, ov.z, cf.NW, w0, lo, hi);
+            scatter_bits(S.clrp, ov.w, cf.NW, w0, lo, hi);
+        }
+    }
+    return make_int2((int)h0.w * (int)cnt, 1);
+}
+
+// Every rule of the env against the warp's planes.  The first two terms of RB
+// rules are evaluated without branches (independent chains the scheduler can
+// overlap); one warp reduction yields the rules that still have a live anchor.
+// Returns (this lane's reward, 1 if this lane wrote an output).
+template <int NA, int RB, bool SM>
+__device__ __forceinline__ int2 warp_rules(const DevConfig &cf, const uint32_t *tab, const WarpSmem &S)
+{
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const unsigned char *pb = reinterpret_cast<const unsigned char *>(S.planes) + q * 8;
+    const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+    const uint32_t total_terms = tab[1];
+    int2 acc = make_int2(0, 0);
+    for (int r0 = 0; r0 < cf.R; r0 += RB) {
+        uint32_t m[RB][NA];
+        uint32_t live = 0;
+#pragma unroll
+        for (int j = 0; j < RB; ++j) {
+            const bool ok = r0 + j < cf.R;
+            const int r = ok ? r0 + j : 0;
+            const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
+            const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
+            const uint32_t *vmr = S.vm + ((h1.z >> (8 * g)) & 0xffu) * cf.NW;
+            const uint32_t np = h0.x, nt = ok ? h0.x + h0.y : 0u;
+            // descriptors of terms 0 and 1 (index clamped to a valid term)
+            const uint32_t t0 = nt > 0 ? h1.x : 0u, t1 = nt > 1 ? h1.x + 1 : t0;
+            const uint2 d0 = total_terms ? ld2<SM>(terms + (size_t)t0 * 4 + g) : make_uint2(0u, 0u);
+            const uint2 d1 = total_terms ? ld2<SM>(terms + (size_t)t1 * 4 + g) : make_uint2(0u, 0u);
+            const uint32_t keep0 = nt > 0 ? 0u : 0xffffffffu;  // no term: pass every anchor
+            const uint32_t keep1 = nt > 1 ? 0u : 0xffffffffu;
+            const uint32_t neg0 = np > 0 ? 0u : 0xffffffffu;
+            const uint32_t neg1 = np > 1 ? 0u : 0xffffffffu;
+            uint32_t any = 0;
+#pragma unroll
+            for (int u = 0; u < NA; ++u) {
+                const int a = q + 8 * u;
+                const uint2 w0 = *reinterpret_cast<const uint2 *>(pb + d0.x + 64 * u);
+                const uint2 w1 = *reinterpret_cast<const uint2 *>(pb + d1.x + 64 * u);
+                const uint32_t x0 = (__funnelshift_r(w0.x, w0.y, d0.y) ^ neg0) | keep0;
+                const uint32_t x1 = (__funnelshift_r(w1.x, w1.y, d1.y) ^ neg1) | keep1;
+                const uint32_t v = (ok && a < cf.NW) ? vmr[a] : 0u;
+                m[j][u] = v & x0 & x1;
+                any |= m[j][u];
+            }
+            live |= (any != 0u ? 1u : 0u) << j;
+        }
+        live = __reduce_or_sync(0xffffffffu, live);
+        while (live) {  // rare: rules with a live anchor after two terms
+            const int j = __ffs(live) - 1;
+            live &= live - 1;
+            Words<NA> mw;
+#pragma unroll
+            for (int jj = 0; jj < RB; ++jj)
+                if (jj == j)
+#pragma unroll
+                    for (int u = 0; u < NA; ++u)
+                        mw.v[u] = m[jj][u];
+            const int2 o = warp_rule_rest<NA, SM>(cf, tab, S, r0 + j, mw);
+            acc.x += o.x;
+            acc.y |= o.y;
+        }
+    }
+    return acc;
+}
+
+__device__ __forceinline__ void warp_fill_actions(const uint8_t *__restrict__ actions, uint64_t seed, int env,
+                                                  int s0, int n_steps, uint8_t *acts, int &warn)
+{
+    const int lane = threadIdx.x & 31;
+    for (int k = lane; k < kActChunk; k += 32) {
+        const int s = s0 + k;
+        if (s < n_steps)
+            acts[s & (kActChunk - 1)] = (uint8_t)action_at(actions, seed, env, s, &warn);
+    }
+}
+
+// next = (D & ~CLEAR) | (~D & SET) in place over the tile planes; SET / CLEAR cleared.
+__device__ __forceinline__ void warp_combine(const DevConfig &cf, const WarpSmem &S)
+{
+    const int lane = threadIdx.x & 31;
+    for (int i = lane; i < cf.C * cf.NW; i += 32) {
+        const int c = i / cf.NW, w = i - c * cf.NW;
+        const uint32_t d = S.planes[c * cf.NWP + w].x, st = S.setp[i], cl = S.clrp[i];
+        S.setp[i] = 0u;
+        S.clrp[i] = 0u;
+        put_word(S.planes, cf.NWP, c, w, (d & ~cl) | (~d & st));
+    }
+}
+
+template <typename CellT, int NA, int RB, bool SM>
+__global__ void __launch_bounds__(32 * kWarpCtaMax)
+expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
+                   const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g,
+                   const CellT *__restrict__ parents, int F, const int32_t *__restrict__ n_parent,
+                   CellT *children, int32_t *rewards, uint8_t *done, uint64_t *hashes)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const long long node = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (node >= (long long)cf.B * F)
+        return;
+    const int env = (int)(node / F);
+    if (n_parent && (int)(node - (long long)env * F) >= n_parent[env])
+        return;  // an empty frontier slot
+    const int lane = threadIdx.x & 31, HW = cf.HW, NW = cf.NW, NWP = cf.NWP, C = cf.C;
+    const WarpSmem S = carve_warp(smem, cf, 5);
+    const int table = cf.rules_per_env ? env : 0;
+    const uint32_t *tab_g = arena + tab_off[table];
+    const uint32_t *tab = SM ? S.rules : tab_g;
+
+    warp_stage(cf, S, vm_g, masks_g, tab_g, tab_off[table + 1] - tab_off[table], SM);
+    warp_cells_to_planes<CellT>(cf, parents + (size_t)node * HW, S.planes, nullptr);
+    __syncwarp();
+    for (int a = 0; a < 5; ++a) {
+        force_plane(cf, S.planes, S.masks, a);
+        __syncwarp();
+        const int2 o = warp_rules<NA, RB, SM>(cf, tab, S);
+        const int rew = __reduce_add_sync(0xffffffffu, o.x);
+        __syncwarp();
+        const bool any = __any_sync(0xffffffffu, o.y != 0);
+        for (int i = lane; i < C * NW; i += 32) {  // child planes
+            const int c = i / NW, w = i - c * NW;
+            const uint32_t d = S.planes[c * NWP + w].x;
+            uint32_t v = d;
+            if (any) {
+                v = (d & ~S.clrp[i]) | (~d & S.setp[i]);
+                S.setp[i] = 0u;
+                S.clrp[i] = 0u;
+            }
+            S.basep[i] = v;
+        }
+        __syncwarp();
+        uint16_t *cells = S.cells + (size_t)a * HW;
+        CellT *dst = children + ((size_t)node * 5 + a) * HW;
+        int goal = 0;
+        for (int p = lane; p < HW; p += 32) {
+            const uint32_t v = gather_cell(cf, nullptr, S.basep, p);
+            cells[p] = (uint16_t)v;
+            dst[p] = (CellT)v;
+            if (cf.ch_goal >= 0)
+                goal |= (int)((v >> cf.ch_goal) & 1u);
+        }
+        const int goal_left = __any_sync(0xffffffffu, goal) || cf.ch_goal < 0;
+        if (lane == 0) {
+            rewards[(size_t)node * 5 + a] = rew;
+            if (done)
+                done[(size_t)node * 5 + a] = (uint8_t)!goal_left;
+        }
+        __syncwarp();
+    }
+    // FNV-1a 64 over the canonical bytes, one lane per child
+    if (lane < 5) {
+        const uint16_t *gc = S.cells + (size_t)lane * HW;
+        uint64_t hsh = 0xcbf29ce484222325ULL;
+        for (int p = 0; p < HW; ++p) {
+            const uint32_t v = gc[p];
+            hsh = (hsh ^ (v & 0xffu)) * 0x100000001b3ULL;
+            if (sizeof(CellT) == 2)
+                hsh = (hsh ^ (v >> 8)) * 0x100000001b3ULL;
+        }
+        hashes[(size_t)node * 5 + lane] = hsh;
+    }
+}
+
+// ============================================================ fast rollout
+// Boards of at most 16 plane words.  One CTA per environment with NWARP warps;
+// warp w owns rules w, w + NWARP, ... (at most RPW).
+//
+// Planes (doubled entries): 0..C-1 tile channels, then C..C+4 the force for
+// actions 0..4 (rebuilt only when the board changes).  A step reads the force
+// of its action by offsetting its force terms by action x plane size; the
+// offset of the next step is loaded before the step's barrier.
+//
+// Each lane holds, per owned rule, the shared addresses, shifts and force
+// flags of the rule's first two present terms for its anchor word, and the
+// word's valid-anchor mask: a rule's per-step test is two 64-bit shared loads,
+// two funnel shifts and one AND.  Rules still live after it continue in the
+// general loop (four terms per warp vote).  A step in which no rule matches
+// changes nothing but the step counter: every thread goes on after a single
+// barrier.  Otherwise all warps combine the SET / CLEAR planes, test the goal,
+// reset, and rebuild the force planes.
+
+struct FastLayout {
+    size_t planes, setp, clrp, basep, vm, masks, ctl, acts, rules, total;
+};
+
+__host__ __device__ inline FastLayout fast_layout(const DevConfig &cf)
+{
+    FastLayout L;
+    const size_t pw = (size_t)cf.C * cf.NW * 4;
+    L.planes = 0;
+    L.setp = align16((size_t)(cf.C + 5) * cf.NWP * 8);
+    L.clrp = align16(L.setp + pw);
+    L.basep = align16(L.clrp + pw);
+    L.vm = align16(L.basep + pw);
+    L.masks = align16(L.vm + (size_t)kShapes * cf.NW * 4);
+    L.ctl = align16(L.masks + (size_t)3 * cf.NW * 4);
+    L.acts = align16(L.ctl + 16 * 4);
+    L.rules = align16(L.acts + kActChunk);
+    L.total = align16(L.rules + (size_t)cf.rule_words * 4);
+    return L;
+}
+
+struct FastSmem {
+    uint2 *planes;
+    uint32_t *setp, *clrp, *basep, *vm, *masks, *rules;
+    int *ctl;  // [0], [1] matches so far at even / odd steps; [2] reward of the step;
+               // [3] warning
+    uint8_t *acts;
+};
+
+// Force planes of actions a0, a0 + stride, ... < 5 from the player plane (one warp).
+static __device__ void force_planes(const DevConfig &cf, uint2 *P, const uint32_t *masks, int a0, int stride)
+{
+    const int lane = threadIdx.x & 31, NW = cf.NW, NWP = cf.NWP;
+    const uint32_t *firstcol = masks, *lastcol = masks + NW, *cellmask = masks + 2 * NW;
+    const uint2 *pl = P + (cf.ch_player >= 0 ? cf.ch_player : 0) * NWP;
+    for (int action = a0; action < 5; action += stride)
+        for (int w = lane; w < NW; w += 32) {
+            uint32_t f = 0;
+            if (cf.ch_player >= 0 && action > 0) {
+                const int n = (action == 1 || action == 3) ? cf.W : 1;
+                const int q = n >> 5, r = n & 31;
+                if (action == 1 || action == 4) {
+                    const uint2 e = pl[w + q];
+                    f = __funnelshift_r(e.x, e.y, r);
+                } else {
+                    const int j = w - q;
+                    if (j >= 1) {
+                        const uint2 e = pl[j - 1];
+                        f = __funnelshift_l(e.x, e.y, r);
+                    } else if (j == 0) {
+                        f = pl[0].x << r;
+                    }
+                }
+                if (action == 2)
+                    f &= ~firstcol[w];
+                else if (action == 4)
+                    f &= ~lastcol[w];
+                f &= cellmask[w];
+            }
+            put_word(P, NWP, cf.C + action, w, f);
+        }
+}
+
+// Terms t0.. of rule r, four per warp vote, then the rule's write.  `m` holds
+// the live anchors so far; force terms read `fdelta` bytes past the action-0
+// force plane.  Returns (this lane's reward, 1 if this lane matched).
+template <int NA, bool SM>
+__device__ __noinline__ int2 fast_rule_rest(const DevConfig &cf, const uint32_t *tab, const FastSmem &S, int r,
+                                            uint32_t t0, uint32_t fdelta, Words<NA> mw)
+{
+    uint32_t *m = mw.v;
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
+    const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
+    const uint32_t force0 = (uint32_t)(cf.C * cf.NWP * 8), force_end = force0 + (uint32_t)(cf.NWP * 8);
+    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)h1.x * 4 + g;
+    const unsigned char *pb = reinterpret_cast<const unsigned char *>(S.planes) + q * 8;
+    const uint32_t np = h0.x, nt = h0.x + h0.y;
+    // a missing term reads the all-zero action-0 force plane, complemented: it passes
+    for (uint32_t t = t0; t < nt; t += 4) {
+        uint2 d[4];
+        uint32_t neg[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t tt = t + j;
+            if (tt < nt) {
+                d[j] = ld2<SM>(tp + 4 * tt);
+                if (d[j].x >= force0 && d[j].x < force_end)
+                    d[j].x += fdelta;
+                neg[j] = tt < np ? 0u : 0xffffffffu;
+            } else {
+                d[j] = make_uint2(force0, 0u);
+                neg[j] = 0xffffffffu;
+            }
+        }
+        uint32_t any = 0;
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            uint32_t x = m[u];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint2 w = *reinterpret_cast<const uint2 *>(pb + d[j].x + 64 * u);
+                x &= __funnelshift_r(w.x, w.y, d[j].y) ^ neg[j];
+            }
+            m[u] = x;
+            any |= x;
+        }
+        if (!__any_sync(0xffffffffu, any != 0u))
+            return make_int2(0, 0);
+    }
+    uint32_t cnt = 0;
+#pragma unroll
+    for (int u = 0; u < NA; ++u)
+        cnt += __popc(m[u]);
+    if (cnt == 0)
+        return make_int2(0, 0);
+    const uint4 *op = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, tab[1])) + (size_t)h1.y * 4 + g;
+    for (uint32_t o = 0; o < h0.z; ++o) {
+        const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            if (!m[u])
+                continue;
+            const int w0 = q + 8 * u + (int)ov.x;
+            const uint32_t lo = m[u] << ov.y;
+            const uint32_t hi = ov.y ? (m[u] >> (32u - ov.y)) : 0u;
+            scatter_bits(S.setp, ov.z, cf.NW, w0, lo, hi);
+            scatter_bits(S.clrp, ov.w, cf.NW, w0, lo, hi);
+        }
+    }
+    return make_int2((int)h0.w * (int)cnt, 1);
+}
+
+__device__ __forceinline__ uint2 lds2(uint32_t addr)
+{
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+// Per-lane register data of one owned rule.
+template <int NA>
+struct FastRule {
+    uint32_t vm[NA];
+    uint32_t a0, a1;  // shared addresses of terms 0 and 1 (force terms: the action-0 plane)
+    uint32_t s0, s1;  // their shifts
+    uint32_t f0, f1;  // 1 for a force term (offset by the step's action), else 0
+};
+
+template <typename CellT, int NA, int NWARP, int RPW, bool SM>
+__global__ void __launch_bounds__(32 * NWARP, NWARP == 8 ? 4 : 7)
+rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
+                    const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
+                    const CellT *__restrict__ init, int32_t *tsteps, int n_steps, uint64_t seed,
+                    const uint8_t *__restrict__ actions, CellT *obs_traj, int32_t *rew_traj,
+                    uint8_t *done_traj, int32_t *rew_sum, uint32_t *status)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const FastLayout L = fast_layout(cf);
+    FastSmem S;
+    S.planes = reinterpret_cast<uint2 *>(smem + L.planes);
+    S.setp = reinterpret_cast<uint32_t *>(smem + L.setp);
+    S.clrp = reinterpret_cast<uint32_t *>(smem + L.clrp);
+    S.basep = reinterpret_cast<uint32_t *>(smem + L.basep);
+    S.vm = reinterpret_cast<uint32_t *>(smem + L.vm);
+    S.masks = reinterpret_cast<uint32_t *>(smem + L.masks);
+    S.ctl = reinterpret_cast<int *>(smem + L.ctl);
+    S.acts = smem + L.acts;
+    S.rules = reinterpret_cast<uint32_t *>(smem + L.rules);
+
+    const int env = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int g = lane >> 3, q = lane & 7;
+    const int HW = cf.HW, NW = cf.NW, NWP = cf.NWP, C = cf.C;
+    const int table = cf.rules_per_env ? env : 0;
+    const uint32_t *tab_g = arena + tab_off[table];
+    const uint32_t *tab = SM ? S.rules : tab_g;
+    const uint32_t plane_bytes = (uint32_t)NWP * 8;
+
+    // ---- stage
+    for (int i = tid; i < (C + 5) * NWP; i += 32 * NWARP)
+        S.planes[i] = make_uint2(0u, 0u);
+    for (int i = tid; i < C * NW; i += 32 * NWARP) {
+        S.setp[i] = 0u;
+        S.clrp[i] = 0u;
+    }
+    for (int i = tid; i < kShapes * NW; i += 32 * NWARP)
+        S.vm[i] = __ldg(vm_g + i);
+    for (int i = tid; i < 3 * NW; i += 32 * NWARP)
+        S.masks[i] = __ldg(masks_g + i);
+    if (SM) {
+        const uint32_t n = tab_off[table + 1] - tab_off[table];
+        const uint4 *src = reinterpret_cast<const uint4 *>(tab_g);
+        uint4 *d = reinterpret_cast<uint4 *>(S.rules);
+        for (uint32_t i = tid; i < n / 4; i += 32 * NWARP)
+            d[i] = __ldg(src + i);
+    }
+    if (tid < 16)
+        S.ctl[tid] = 0;
+    __syncthreads();
+    for (int k = tid; k < kActChunk; k += 32 * NWARP)
+        if (k < n_steps)
+            S.acts[k] = (uint8_t)action_at(actions, seed, env, k, S.ctl + 3);
+    {
+        const CellT *src = cur + (size_t)env * HW, *isrc = init + (size_t)env * HW;
+        for (int base = 0; base < HW; base += 32 * NWARP) {
+            const int p = base + tid;
+            const uint32_t v = p < HW ? (uint32_t)src[p] : 0u;
+            const uint32_t vi = p < HW ? (uint32_t)isrc[p] : 0u;
+            const int w = p >> 5;
+            for (int c = 0; c < C; ++c) {
+                const uint32_t bits = __ballot_sync(0xffffffffu, (v >> c) & 1u);
+                const uint32_t ibits = __ballot_sync(0xffffffffu, (vi >> c) & 1u);
+                if (lane == 0 && w < NW) {
+                    put_word(S.planes, NWP, c, w, bits);
+                    S.basep[c * NW + w] = ibits;
+                }
+            }
+        }
+    }
+    __syncthreads();
+    force_planes(cf, S.planes, S.masks, warp, NWARP);
+
+    // ---- per-lane register data of the owned rules
+    FastRule<NA> fr[RPW];
+    uint32_t slow = 0;
+    {
+        const uint32_t base = (uint32_t)__cvta_generic_to_shared(S.planes) + q * 8;
+        const uint32_t force0 = (uint32_t)C * plane_bytes;
+        const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+#pragma unroll
+        for (int k = 0; k < RPW; ++k) {
+            const int r = warp + k * NWARP;
+            FastRule<NA> &f = fr[k];
+#pragma unroll
+            for (int u = 0; u < NA; ++u)
+                f.vm[u] = 0;
+            f.a0 = f.a1 = base;
+            f.s0 = f.s1 = 0;
+            f.f0 = f.f1 = 0;
+            if (r < cf.R) {
+                const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
+                const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
+                const uint32_t *vmr = S.vm + ((h1.z >> (8 * g)) & 0xffu) * NW;
+#pragma unroll
+                for (int u = 0; u < NA; ++u) {
+                    const int a = q + 8 * u;
+                    f.vm[u] = a < NW ? vmr[a] : 0u;
+                }
+                if (h0.x >= 2) {
+                    const uint2 d0 = ld2<SM>(terms + (size_t)h1.x * 4 + g);
+                    const uint2 d1 = ld2<SM>(terms + (size_t)(h1.x + 1) * 4 + g);
+                    f.a0 = base + d0.x;
+                    f.a1 = base + d1.x;
+                    f.s0 = d0.y;
+                    f.s1 = d1.y;
+                    f.f0 = d0.x >= force0 && d0.x < force0 + plane_bytes;
+                    f.f1 = d1.x >= force0 && d1.x < force0 + plane_bytes;
+                } else {
+                    slow |= 1u << k;  // fewer than two present terms: the general loop from term 0
+                }
+            }
+        }
+    }
+    int t = tsteps[env];
+    int goal_left;
+    {
+        int gl = cf.ch_goal < 0;
+        if (cf.ch_goal >= 0)
+            for (int w = lane; w < NW; w += 32)
+                gl |= S.planes[cf.ch_goal * NWP + w].x != 0u;
+        goal_left = __syncthreads_or(gl);  // also publishes the force planes
+    }
+
+    int seen0 = 0, seen1 = 0, sum = 0;
+    uint32_t fdelta = (uint32_t)S.acts[0] * plane_bytes;
+    for (int s = 0; s < n_steps; ++s) {
+        const int par = s & 1;
+        // ---- first pair of every owned rule from registers
+        uint32_t m[RPW][NA];
+        uint32_t anyall = 0;
+#pragma unroll
+        for (int k = 0; k < RPW; ++k) {
+            const FastRule<NA> &f = fr[k];
+            const uint32_t a0 = f.a0 + f.f0 * fdelta, a1 = f.a1 + f.f1 * fdelta;
+#pragma unroll
+            for (int u = 0; u < NA; ++u) {
+                const uint2 w0 = lds2(a0 + 64 * u), w1 = lds2(a1 + 64 * u);
+                m[k][u] = f.vm[u] & __funnelshift_r(w0.x, w0.y, f.s0) & __funnelshift_r(w1.x, w1.y, f.s1);
+                anyall |= m[k][u];
+            }
+        }
+        if (__any_sync(0xffffffffu, anyall != 0u) || slow) {  // rare: some rule still live
+            int2 acc = make_int2(0, 0);
+#pragma unroll
+            for (int k = 0; k < RPW; ++k) {
+                const bool from0 = (slow >> k) & 1u;
+                uint32_t any = 0;
+                Words<NA> mw;
+#pragma unroll
+                for (int u = 0; u < NA; ++u) {
+                    mw.v[u] = from0 ? fr[k].vm[u] : m[k][u];
+                    any |= mw.v[u];
+                }
+                if (!__any_sync(0xffffffffu, any != 0u))
+                    continue;
+                const int2 o = fast_rule_rest<NA, SM>(cf, tab, S, warp + k * NWARP, from0 ? 0u : 2u, fdelta, mw);
+                acc.x += o.x;
+                acc.y |= o.y;
+            }
+            const int wrew = __reduce_add_sync(0xffffffffu, acc.x);
+            if (__any_sync(0xffffffffu, acc.y != 0) && lane == 0) {
+                atomicAdd(S.ctl + 2, wrew);
+                atomicAdd(S.ctl + par, 1);  // read after this step's barrier, next written two steps on
+            }
+        }
+        // actions [s + 128, s + 256) into ring slots no step in [s, s + 128) reads
+        if (warp == NWARP - 1 && s > 0 && (s & (kActChunk / 2 - 1)) == 0)
+            for (int k = lane; k < kActChunk / 2; k += 32)
+                if (s + kActChunk / 2 + k < n_steps)
+                    S.acts[(s + kActChunk / 2 + k) & (kActChunk - 1)] =
+                        (uint8_t)action_at(actions, seed, env, s + kActChunk / 2 + k, S.ctl + 3);
+        const uint32_t fdelta_next = (uint32_t)S.acts[(s + 1) & (kActChunk - 1)] * plane_bytes;
+        __syncthreads();
+
+        const int matches = S.ctl[par];
+        t += 1;
+        int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+        if (matches == (par ? seen1 : seen0) && !(done && cf.auto_reset)) {
+            // nothing changed: no reward, same board
+            if (tid == 0) {
+                if (rew_traj)
+                    rew_traj[(size_t)s * cf.B + env] = 0;
+                if (done_traj)
+                    done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
+            }
+        } else {
+            if (par)
+                seen1 = matches;
+            else
+                seen0 = matches;
+            // combine, all warps: a bit changes where any match asks for it; one
+            // thread per word, so the goal test of the new board comes with it
+            int gl = cf.ch_goal < 0;
+            for (int i = tid; i < C * NW; i += 32 * NWARP) {
+                const int c = i / NW, w = i - c * NW;
+                uint32_t d = S.planes[c * NWP + w].x;
+                const uint32_t st = S.setp[i], cl = S.clrp[i];
+                if (st | cl) {
+                    S.setp[i] = 0u;
+                    S.clrp[i] = 0u;
+                    d = (d & ~cl) | (~d & st);
+                    put_word(S.planes, NWP, c, w, d);
+                }
+                if (c == cf.ch_goal)
+                    gl |= d != 0u;
+            }
+            goal_left = __syncthreads_or(gl);
+            done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+            if (done && cf.auto_reset) {
+                for (int i = tid; i < C * NW; i += 32 * NWARP) {
+                    const int c = i / NW, w = i - c * NW;
+                    put_word(S.planes, NWP, c, w, S.basep[i]);
+                }
+                t = 0;
+                gl = cf.ch_goal < 0;
+                if (cf.ch_goal >= 0)
+                    for (int w = tid; w < NW; w += 32 * NWARP)
+                        gl |= S.basep[cf.ch_goal * NW + w] != 0u;
+                goal_left = __syncthreads_or(gl);
+            }
+            force_planes(cf, S.planes, S.masks, warp, NWARP);
+            if (tid == 0) {
+                const int rew = S.ctl[2];
+                sum += rew;
+                S.ctl[2] = 0;
+                if (rew_traj)
+                    rew_traj[(size_t)s * cf.B + env] = rew;
+                if (done_traj)
+                    done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
+            }
+            __syncthreads();
+        }
+        if (obs_traj) {
+            CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
+            for (int p = tid; p < HW; p += 32 * NWARP)
+                dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+        }
+        fdelta = fdelta_next;
+    }
+    CellT *dst = cur + (size_t)env * HW;
+    for (int p = tid; p < HW; p += 32 * NWARP)
+        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+    if (tid == 0) {
+        tsteps[env] = t;
+        if (rew_sum)
+            rew_sum[env] = sum;
+        if (S.ctl[3])
+            atomicOr(status + 1, kWarnAction);
+    }
+}
+
 template <typename CellT>
 __global__ void __launch_bounds__(kThreads)
 reset_kernel(DevConfig cf, const uint32_t *__restrict__ cum_all, uint64_t seed, CellT *cur,
@@ -684,7 +1432,7 @@ __device__ __forceinline__ bool key_less(const Key128 &a, const Key128 &b)
 }
 
 // Block-wide bitonic sort of n2 (power of two) keys in shared memory, ascending.
-__device__ void bitonic_sort(Key128 *keys, int n2)
+static __device__ void bitonic_sort(Key128 *keys, int n2)
 {
     for (int k = 2; k <= n2; k <<= 1)
         for (int j = k >> 1; j > 0; j >>= 1) {
@@ -853,7 +1601,7 @@ select_kernel(DevConfig cf, int cap, int parity, int F, const int32_t *__restric
         n_visited[b] = nv + take;
 }
 
-// ------------------------------------------------------------ launchers
+// ------------------------------------------------------------ host helpers
 inline size_t select_smem_bytes(int F)
 {
     int n2 = 1;
@@ -872,142 +1620,13 @@ inline int anchor_slots(int NW)
     return na;
 }
 
-#define AV_FOR_NA(MACRO, CELL) MACRO(CELL, 1) MACRO(CELL, 2) MACRO(CELL, 4) MACRO(CELL, 8) MACRO(CELL, 16)
+// Paths: cf.path 0 = choose, 1 = block per env, 3 = fast rollout.
+// Rollouts: the fast kernel for boards of at most 16 plane words and <= 64
+// rules unless the block path is forced; expansion: one warp per parent for
+// boards of at most 16 plane words unless the block path is forced.
+inline bool use_fast_rollout(const DevConfig &cf) { return cf.NA <= 2 && cf.R <= 64 && cf.path != 1; }
+inline bool use_warp_expand(const DevConfig &cf) { return cf.NA <= 2 && cf.path != 1; }
 
-inline cudaError_t configure_kernels(const DevConfig &cf)
-{
-    (void)cf;
-    const int big = 200 * 1024;
-    cudaError_t e = cudaSuccess;
-    auto set = [&](const void *fn) {
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, big);
-    };
-#define AV_SET(CELL, NA)                                       \
-    set((const void *)rollout_kernel<CELL, NA, true>);         \
-    set((const void *)rollout_kernel<CELL, NA, false>);        \
-    set((const void *)expand_kernel<CELL, NA, true>);          \
-    set((const void *)expand_kernel<CELL, NA, false>);
-    AV_FOR_NA(AV_SET, uint8_t)
-    AV_FOR_NA(AV_SET, uint16_t)
-#undef AV_SET
-    set((const void *)reset_kernel<uint8_t>);
-    set((const void *)reset_kernel<uint16_t>);
-    set((const void *)select_kernel<uint8_t>);
-    set((const void *)select_kernel<uint16_t>);
-    return e;
-}
-
-template <typename CellT, int NA>
-void rollout_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
-               const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
-               const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj,
-               int32_t *rew_sum, uint32_t *status, cudaStream_t st)
-{
-    if (cf.rule_words > 0)
-        rollout_kernel<CellT, NA, true><<<cf.B, kThreads, step_smem(cf, 0).total, st>>>(
-            cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
-            (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
-    else
-        rollout_kernel<CellT, NA, false><<<cf.B, kThreads, step_smem(cf, 0).total, st>>>(
-            cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
-            (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
-}
-
-inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
-                           const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
-                           int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
-                           int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
-                           cudaStream_t st)
-{
-#define AV_CASE(CELL, NA)                                                                              \
-    case NA:                                                                                          \
-        rollout_t<CELL, NA>(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions,      \
-                            obs_traj, rew_traj, done_traj, rew_sum, status, st);                      \
-        break;
-    if (cf.cell_bytes == 1) {
-        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint8_t) }
-    } else {
-        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint16_t) }
-    }
-#undef AV_CASE
-}
-
-template <typename CellT, int NA>
-void expand_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
-              const uint32_t *masks, const void *parents, int F, const int32_t *n_parent, void *children,
-              int32_t *rewards, uint8_t *done, uint64_t *hashes, cudaStream_t st)
-{
-    if (cf.rule_words > 0)
-        expand_kernel<CellT, NA, true><<<(unsigned)(cf.B * F), kThreads, step_smem(cf, 5).total, st>>>(
-            cf, arena, tab_off, vm, masks, (const CellT *)parents, F, n_parent, (CellT *)children, rewards,
-            done, hashes);
-    else
-        expand_kernel<CellT, NA, false><<<(unsigned)(cf.B * F), kThreads, step_smem(cf, 5).total, st>>>(
-            cf, arena, tab_off, vm, masks, (const CellT *)parents, F, n_parent, (CellT *)children, rewards,
-            done, hashes);
-}
-
-inline void launch_expand(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
-                          const uint32_t *vm, const uint32_t *masks, const void *parents, int F,
-                          const int32_t *n_parent, void *children, int32_t *rewards, uint8_t *done,
-                          uint64_t *hashes, cudaStream_t st)
-{
-#define AV_CASE(CELL, NA)                                                                              \
-    case NA:                                                                                          \
-        expand_t<CELL, NA>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards,    \
-                           done, hashes, st);                                                         \
-        break;
-    if (cf.cell_bytes == 1) {
-        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint8_t) }
-    } else {
-        switch (cf.NA) { AV_FOR_NA(AV_CASE, uint16_t) }
-    }
-#undef AV_CASE
-}
-
-inline void launch_reset(const DevConfig &cf, const uint32_t *cum, uint64_t seed, void *cur, void *init,
-                         int32_t *t, void *obs, cudaStream_t st)
-{
-    const size_t sm = align16((size_t)cf.HW * 2);
-    if (cf.cell_bytes == 1)
-        reset_kernel<uint8_t><<<cf.B, kThreads, sm, st>>>(cf, cum, seed, (uint8_t *)cur, (uint8_t *)init, t,
-                                                         (uint8_t *)obs);
-    else
-        reset_kernel<uint16_t><<<cf.B, kThreads, sm, st>>>(cf, cum, seed, (uint16_t *)cur, (uint16_t *)init,
-                                                          t, (uint16_t *)obs);
-}
-
-inline void launch_search_init(const DevConfig &cf, int cap, const void *roots, uint64_t *root_hash,
-                               uint8_t *root_live, uint64_t *visited, int32_t *n_visited, cudaStream_t st)
-{
-    const unsigned grid = (unsigned)((cf.B + 127) / 128);
-    if (cf.cell_bytes == 1)
-        search_init_kernel<uint8_t><<<grid, 128, 0, st>>>(cf, cap, (const uint8_t *)roots, root_hash, root_live,
-                                                         visited, n_visited);
-    else
-        search_init_kernel<uint16_t><<<grid, 128, 0, st>>>(cf, cap, (const uint16_t *)roots, root_hash,
-                                                          root_live, visited, n_visited);
-}
-
-inline void launch_select(const DevConfig &cf, int cap, int parity, int F, const int32_t *n_parent,
-                          const int32_t *parent_cum, const uint8_t *parent_live, const void *cand_grids,
-                          const int32_t *cand_reward, const uint8_t *cand_done, const uint64_t *cand_hash,
-                          int k, void *next_grids, int32_t *next_cum, uint64_t *next_hash,
-                          uint8_t *next_live, int32_t *n_next, uint64_t *visited, int32_t *n_visited,
-                          uint32_t *status, cudaStream_t st)
-{
-    const size_t sm = select_smem_bytes(F);
-    if (cf.cell_bytes == 1)
-        select_kernel<uint8_t><<<cf.B, kThreads, sm, st>>>(
-            cf, cap, parity, F, n_parent, parent_cum, parent_live, (const uint8_t *)cand_grids, cand_reward,
-            cand_done, cand_hash, k, (uint8_t *)next_grids, next_cum, next_hash, next_live, n_next, visited,
-            n_visited, status);
-    else
-        select_kernel<uint16_t><<<cf.B, kThreads, sm, st>>>(
-            cf, cap, parity, F, n_parent, parent_cum, parent_live, (const uint16_t *)cand_grids, cand_reward,
-            cand_done, cand_hash, k, (uint16_t *)next_grids, next_cum, next_hash, next_live, n_next, visited,
-            n_visited, status);
-}
+constexpr int kDynSmemLimit = 200 * 1024;
 
 }  // namespace av

@@ -1,0 +1,75 @@
+// launch.h -- host-side launchers of libautoverse.so's kernels.  Each group of
+// kernels is instantiated in its own translation unit (k_*.cu) so that the
+// library builds in parallel.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "kernels.cuh"
+
+namespace av {
+
+// Allow each group's kernels the dynamic shared memory they need.
+cudaError_t configure_fast_u8();
+cudaError_t configure_fast_u16();
+cudaError_t configure_block();
+cudaError_t configure_expand();
+cudaError_t configure_search();
+
+void launch_rollout_fast_u8(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
+                            const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
+                            int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
+                            int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                            cudaStream_t st);
+void launch_rollout_fast_u16(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
+                             const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
+                             int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
+                             int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                             cudaStream_t st);
+void launch_rollout_block(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
+                          const uint32_t *vm, const uint32_t *masks, void *cur, const void *init, int32_t *t,
+                          int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
+                          int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                          cudaStream_t st);
+void launch_expand(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+                   const uint32_t *masks, const void *parents, int F, const int32_t *n_parent, void *children,
+                   int32_t *rewards, uint8_t *done, uint64_t *hashes, cudaStream_t st);
+void launch_reset(const DevConfig &cf, const uint32_t *cum, uint64_t seed, void *cur, void *init, int32_t *t,
+                  void *obs, cudaStream_t st);
+void launch_search_init(const DevConfig &cf, int cap, const void *roots, uint64_t *root_hash,
+                        uint8_t *root_live, uint64_t *visited, int32_t *n_visited, cudaStream_t st);
+void launch_select(const DevConfig &cf, int cap, int parity, int F, const int32_t *n_parent,
+                   const int32_t *parent_cum, const uint8_t *parent_live, const void *cand_grids,
+                   const int32_t *cand_reward, const uint8_t *cand_done, const uint64_t *cand_hash, int k,
+                   void *next_grids, int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live,
+                   int32_t *n_next, uint64_t *visited, int32_t *n_visited, uint32_t *status, cudaStream_t st);
+
+inline cudaError_t configure_kernels()
+{
+    cudaError_t e = configure_fast_u8();
+    if (e == cudaSuccess) e = configure_fast_u16();
+    if (e == cudaSuccess) e = configure_block();
+    if (e == cudaSuccess) e = configure_expand();
+    if (e == cudaSuccess) e = configure_search();
+    return e;
+}
+
+inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
+                           const uint32_t *vm, const uint32_t *masks, void *cur, const void *init, int32_t *t,
+                           int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
+                           int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                           cudaStream_t st)
+{
+    if (use_fast_rollout(cf) && cf.cell_bytes == 1)
+        launch_rollout_fast_u8(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
+                               rew_traj, done_traj, rew_sum, status, st);
+    else if (use_fast_rollout(cf))
+        launch_rollout_fast_u16(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
+                                rew_traj, done_traj, rew_sum, status, st);
+    else
+        launch_rollout_block(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
+                             rew_traj, done_traj, rew_sum, status, st);
+}
+
+}  // namespace av

@@ -210,3 +210,53 @@ def test_dense_matches_stress_apply():
     np.testing.assert_array_equal(to_np(res["rew"]), ref["rew"])
     assert np.abs(ref["rew"]).sum() > 1000
     env.close()
+
+
+# ------------------------------------------------- both kernel paths
+@pytest.mark.parametrize("path", ["block", "fast", "fast8"])
+@pytest.mark.parametrize("key,batch,steps", [(1, 3, 60), (2, 9, 70), (3, 7, 230), (4, 4, 30)])
+def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
+    monkeypatch.setenv("AV_KERNEL_PATH", path.rstrip("8"))
+    if path.endswith("8"):
+        monkeypatch.setenv("AV_FAST_WARPS", "8")
+    wl = wk.WORKLOADS[key].scaled(batch=batch)
+    env, cfg, rules, cum = make(wl, 11 + key)
+    s = wk.seeds(11 + key)
+    g0 = to_np(env.reset(s["reset"]))
+    res = env.rollout(steps, s["actions"], trajectory=True)
+    ref = _oracle_rollout(cfg, rules, g0, np.arange(batch), steps, s["actions"])
+    np.testing.assert_array_equal(to_np(res["obs"]), ref["obs"])
+    np.testing.assert_array_equal(to_np(res["rew"]), ref["rew"])
+    np.testing.assert_array_equal(to_np(res["done"]), ref["done"])
+    g, t = env.get_state()
+    np.testing.assert_array_equal(to_np(t), ref["t"])
+    env.close()
+
+
+@pytest.mark.parametrize("path", ["block", "fast", "fast8"])
+@pytest.mark.parametrize("H,W,C,shapes,R", [
+    (1, 1, 1, ((1, 1),), 2),
+    (7, 9, 3, ((3, 3), (5, 5), (1, 4)), 4),
+    (5, 5, 16, ((5, 5), (4, 2)), 2),
+    (2, 64, 9, ((1, 5), (2, 2)), 3),
+    (20, 21, 6, ((3, 3), (2, 4)), 9),  # 420 cells: two anchor words per lane
+    (16, 16, 5, ((1, 1), (1, 2)), 40),  # many rules: several per warp
+])
+def test_both_kernel_paths_edges(monkeypatch, path, H, W, C, shapes, R):
+    monkeypatch.setenv("AV_KERNEL_PATH", path.rstrip("8"))
+    if path.endswith("8"):
+        monkeypatch.setenv("AV_FAST_WARPS", "8")
+    wl = wk.Workload(0, "edge", 5, H, W, C, R, shapes, 0.1, 0.06, 0.2, 0.2, -2, 2,
+                     steps=15, max_steps=6, auto_reset=1)
+    _, rules, _ = wk.make(wl, 21)
+    g0 = wk.random_grids(9, 5, H, W, C, density=0.45)
+    if C > 2:
+        g0[:, H // 2, W // 2] |= 1 << 2
+    env, cfg, _, _ = make(wl, 0, rules=rules, cum=None)
+    env.set_state(to_dev(g0), set_as_init=True)
+    res = env.rollout(15, 123, trajectory=True)
+    ref = oracle.rollout(cfg, rules, g0, g0, np.zeros(5), 15, 123, trajectory=True)
+    np.testing.assert_array_equal(to_np(res["obs"]), ref["obs"])
+    np.testing.assert_array_equal(to_np(res["rew"]), ref["rew"])
+    np.testing.assert_array_equal(to_np(res["done"]), ref["done"])
+    env.close()

@@ -140,3 +140,18 @@ def test_visited_overflow_reports_device_error():
     assert ei.value.status == av.AV_EDEVICE
     env.sync()  # the status is cleared once reported
     env.close()
+
+
+@pytest.mark.parametrize("path", ["block", "default"])
+def test_expand_both_kernel_paths(monkeypatch, path):
+    monkeypatch.setenv("AV_KERNEL_PATH", path)
+    wl = wk.WORKLOADS[3].scaled(batch=5)
+    env, cfg, rules, cum = make(wl, 6)
+    parents = _parents(wl, cfg, rules, cum, 11, 17)
+    ch, rew, done, hsh = env.expand(to_dev(parents))
+    ech, erew, edone, ehsh = oracle.expand(cfg, rules, parents)
+    np.testing.assert_array_equal(to_np(ch), ech)
+    np.testing.assert_array_equal(to_np(rew), erew)
+    np.testing.assert_array_equal(to_np(done), edone)
+    np.testing.assert_array_equal(to_np(hsh, "hash"), ehsh)
+    env.close()
