@@ -145,29 +145,43 @@ void turn_position(int h, int w, int g, int &i, int &k)
 // Compile one rule table into the layout read by the kernels (kernels.cuh,
 // "Rule table layout").  The term order is chosen once on the base pattern
 // and carried through every rotation, so the four rotations of a rule run
-// the same loop: an exclusive pair of present tile channels first (see
-// below), then a present force term, positions with more present channels,
-// the player channel, higher channels; absent entries last.  Any order gives
-// the same result; a selective order lets evaluation stop early.
-void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32_t> &arena)
+// the same loop.  Any order gives the same result; a selective order lets
+// evaluation stop early.  Present terms: an exclusive pair of present tile
+// channels first (see below), then a present force term, positions with more
+// present channels, the player channel, then rarer channels.  Absent terms
+// follow: first those at positions with no present tile channel (at a
+// position whose tile is already fixed by a present term, an absent tile
+// channel almost always holds), the most common channels first.  `density`
+// (C entries, or null) is each tile channel's share of cells in the initial
+// maps; without it every tile channel counts as equally common.
+void compile_table(const av_rule *rules, const DevConfig &cf, const double *density, std::vector<uint32_t> &arena)
 {
     const size_t base = arena.size();
     const int R = cf.R;
     std::vector<uint32_t> hdr(8 * (size_t)R, 0), terms, outs;
     uint32_t n_terms = 0, n_outs = 0;
+    // how common a channel is on a cell: the force and the player mark one cell
+    auto common = [&](int c) -> double {
+        if (c == cf.C || c == cf.ch_player)
+            return 1.0 / cf.HW;
+        return density ? density[c] : 1.0 / cf.C;
+    };
     for (int r = 0; r < R; ++r) {
         const Pat p = from_record(rules[r]);
-        struct BT { int i, k, c, neg, key0, key1; };
+        struct BT { int i, k, c, neg, key0, key1; double dens; };
         std::vector<BT> pres, absn;
         for (int i = 0; i < p.h; ++i)
             for (int k = 0; k < p.w; ++k) {
                 const int e = i * p.w + k;
                 const int npos = __builtin_popcount(p.pres[e]);
+                uint32_t tiles = p.pres[e] & ((1u << cf.C) - 1u);
+                if (cf.ch_player >= 0)
+                    tiles &= ~(1u << cf.ch_player);
                 for (int c = 0; c <= cf.C; ++c) {
                     const int rank = c == cf.C ? 2 : (c == cf.ch_player ? 1 : 0);
                     const int key0 = c == cf.C ? 100 + npos : npos;  // a present force term first
-                    if ((p.pres[e] >> c) & 1u) pres.push_back({i, k, c, 0, key0, rank});
-                    if ((p.abs_[e] >> c) & 1u) absn.push_back({i, k, c, 1, 0, 0});
+                    if ((p.pres[e] >> c) & 1u) pres.push_back({i, k, c, 0, key0, rank, common(c)});
+                    if ((p.abs_[e] >> c) & 1u) absn.push_back({i, k, c, 1, tiles ? 1 : 0, 0, common(c)});
                 }
             }
         std::stable_sort(pres.begin(), pres.end(), [](const BT &a, const BT &b) {
@@ -175,7 +189,12 @@ void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32
             if (a.key0 > 1 && a.key0 < 100 && a.i * 8 + a.k != b.i * 8 + b.k)
                 return a.i * 8 + a.k < b.i * 8 + b.k;  // keep a position's present terms together
             if (a.key1 != b.key1) return a.key1 > b.key1;
+            if (a.dens != b.dens) return a.dens < b.dens;
             return a.c > b.c;
+        });
+        std::stable_sort(absn.begin(), absn.end(), [](const BT &a, const BT &b) {
+            if (a.key0 != b.key0) return a.key0 < b.key0;  // positions without a present tile first
+            return a.dens > b.dens;
         });
         // An exclusive pair leads when the rule has one: two present tile
         // channels (neither the player's) at one position.  Initial maps hold
@@ -196,7 +215,7 @@ void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32
                     found = 1;
                 }
             }
-        uint32_t *hd = &hdr[8 * (size_t)r];
+    uint32_t *hd = &hdr[8 * (size_t)r];
         hd[0] = (uint32_t)pres.size();
         hd[1] = (uint32_t)absn.size();
         hd[3] = (uint32_t)p.reward;
@@ -216,7 +235,7 @@ void compile_table(const av_rule *rules, const DevConfig &cf, std::vector<uint32
                 turn_position(p.h, p.w, g, i, k);
                 const int s = i * cf.W + k;
                 terms.push_back((uint32_t)((t.c * cf.NWP + (s >> 5)) * 8));
-                terms.push_back((uint32_t)(s & 31));
+                terms.push_back((uint32_t)(s & 31) | (t.neg ? kTermAbsent : 0u));
             }
             ++n_terms;
         }
@@ -382,20 +401,44 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     cf.cum_per_env = cfg->cum_per_env;
     cf.cell_bytes = cfg->C <= 8 ? 1 : 2;
     // Kernel path override, for testing every path on the same shapes:
-    // AV_KERNEL_PATH=block forces the one-CTA-per-env kernels (default: the fast
-    // rollout and one-warp-per-parent expansion for boards of at most 16 plane
-    // words); AV_FAST_WARPS=8 runs the fast rollout with 8 warps per env.
+    // AV_KERNEL_PATH selects a rollout kernel for tests and measurements:
+    // block (one CTA per env), fast (several warps per env) or warp (one warp
+    // per env); by default the library chooses.  AV_FAST_WARPS=8 runs the fast
+    // rollout with 8 warps per env.
     if (const char *path = getenv("AV_KERNEL_PATH"))
-        cf.path = strcmp(path, "block") == 0 ? 1 : 0;
+        cf.path = strcmp(path, "block") == 0 ? 1 : strcmp(path, "fast") == 0 ? 2 : strcmp(path, "warp") == 0 ? 3 : 0;
     if (const char *fw = getenv("AV_FAST_WARPS"))
         cf.fast_warps = atoi(fw) == 8 ? 8 : 4;
     h->grid_bytes = (size_t)cf.HW * cf.cell_bytes;
 
     std::vector<uint32_t> arena, tab_off((size_t)n_tables + 1);
     uint32_t max_words = 0;
+    // tile-channel densities of the initial maps, per table, for the term order
+    std::vector<double> density;
+    if (cfg->init_cum) {
+        const int n_cum = cfg->cum_per_env ? cf.B : 1;
+        density.assign((size_t)n_cum * cf.C, 0.0);
+        for (int e = 0; e < n_cum; ++e)
+            for (int c = 0; c < cf.C; ++c) {
+                const uint32_t hi = cfg->init_cum[(size_t)e * cf.C + c];
+                const uint32_t lo = c ? cfg->init_cum[(size_t)e * cf.C + c - 1] : 0u;
+                density[(size_t)e * cf.C + c] = hi > lo ? (double)(hi - lo) / 16777216.0 : 0.0;
+            }
+        if (n_cum > 1 && n_tables == 1) {  // one shared table: the mean over environments
+            for (int e = 1; e < n_cum; ++e)
+                for (int c = 0; c < cf.C; ++c)
+                    density[c] += density[(size_t)e * cf.C + c];
+            density.resize(cf.C);
+            for (double &d : density)
+                d /= n_cum;
+        }
+    }
     for (int t = 0; t < n_tables; ++t) {
         tab_off[t] = (uint32_t)arena.size();
-        compile_table(rules + (size_t)t * cfg->n_rules, cf, arena);
+        const double *dens = nullptr;
+        if (!density.empty())
+            dens = density.data() + (density.size() > (size_t)cf.C && n_tables == cf.B ? (size_t)t * cf.C : 0);
+        compile_table(rules + (size_t)t * cfg->n_rules, cf, dens, arena);
         max_words = std::max(max_words, (uint32_t)arena.size() - tab_off[t]);
     }
     tab_off[n_tables] = (uint32_t)arena.size();

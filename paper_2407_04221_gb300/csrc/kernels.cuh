@@ -28,7 +28,8 @@
 //                        first term, first output, shapes (rotation g in byte g:
 //                        (h'-1)*5 + (w'-1)), 0
 //   terms   (uint2, 16-byte aligned, [term][rotation]):
-//           (byte offset of plane entry c*NWP + (s >> 5), s & 31)
+//           (byte offset of plane entry c*NWP + (s >> 5), s & 31 | kTermAbsent
+//           for an absent term; funnel shifts use only the low five bits)
 //   outputs (uint4, [output][rotation]): (s >> 5, s & 31, set bits, clear bits)
 #pragma once
 
@@ -48,6 +49,7 @@ constexpr int kActChunk = 256;  // actions drawn ahead, per CTA
 constexpr int kMaxSmemRuleWords = 8192;  // stage a rule table in shared memory up to 32 KiB
 constexpr uint32_t kStatusVisitedOverflow = 1u;
 constexpr uint32_t kWarnAction = 1u;
+constexpr uint32_t kTermAbsent = 0x80000000u;  // flag in a term's shift word
 
 struct DevConfig {
     int B, H, W, C, HW, NW, NWP, NA;  // NW plane words; NWP doubled entries per plane; NA words per lane
@@ -55,7 +57,7 @@ struct DevConfig {
     int ch_player, ch_goal, ch_empty, ch_wall, border_wall, cum_per_env;
     int cell_bytes;
     int rule_words;  // largest rule table (words) when tables are staged in shared memory, else 0
-    int path;        // 0: choose; 1: one CTA per env (block) kernels forced
+    int path;        // 0: choose; 1: block kernels; 2: fast rollout; 3: one warp per env
     int fast_warps;  // fast rollout: warps per environment (4, or 8 when set to 8)
 };
 
@@ -910,7 +912,7 @@ __host__ __device__ inline FastLayout fast_layout(const DevConfig &cf)
     FastLayout L;
     const size_t pw = (size_t)cf.C * cf.NW * 4;
     L.planes = 0;
-    L.setp = align16((size_t)(cf.C + 5) * cf.NWP * 8);
+    L.setp = align16((size_t)(cf.C + 7) * cf.NWP * 8);
     L.clrp = align16(L.setp + pw);
     L.basep = align16(L.clrp + pw);
     L.vm = align16(L.basep + pw);
@@ -930,8 +932,10 @@ struct FastSmem {
     uint8_t *acts;
 };
 
-// Force planes of actions a0, a0 + stride, ... < 5 from the player plane (one warp).
-static __device__ void force_planes(const DevConfig &cf, uint2 *P, const uint32_t *masks, int a0, int stride)
+// Force planes of actions a0, a0 + stride, ... < 5 from the player plane (one
+// warp), into planes first + action.
+static __device__ void force_planes(const DevConfig &cf, uint2 *P, const uint32_t *masks, int a0, int stride,
+                                    int first)
 {
     const int lane = threadIdx.x & 31, NW = cf.NW, NWP = cf.NWP;
     const uint32_t *firstcol = masks, *lastcol = masks + NW, *cellmask = masks + 2 * NW;
@@ -960,7 +964,7 @@ static __device__ void force_planes(const DevConfig &cf, uint2 *P, const uint32_
                     f &= ~lastcol[w];
                 f &= cellmask[w];
             }
-            put_word(P, NWP, cf.C + action, w, f);
+            put_word(P, NWP, first + action, w, f);
         }
 }
 
@@ -1080,7 +1084,7 @@ rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
     const uint32_t plane_bytes = (uint32_t)NWP * 8;
 
     // ---- stage
-    for (int i = tid; i < (C + 5) * NWP; i += 32 * NWARP)
+    for (int i = tid; i < (C + 6) * NWP; i += 32 * NWARP)
         S.planes[i] = make_uint2(0u, 0u);
     for (int i = tid; i < C * NW; i += 32 * NWARP) {
         S.setp[i] = 0u;
@@ -1121,7 +1125,7 @@ rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
         }
     }
     __syncthreads();
-    force_planes(cf, S.planes, S.masks, warp, NWARP);
+    force_planes(cf, S.planes, S.masks, warp, NWARP, cf.C);
 
     // ---- per-lane register data of the owned rules
     FastRule<NA> fr[RPW];
@@ -1271,7 +1275,7 @@ rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
                         gl |= S.basep[cf.ch_goal * NW + w] != 0u;
                 goal_left = __syncthreads_or(gl);
             }
-            force_planes(cf, S.planes, S.masks, warp, NWARP);
+            force_planes(cf, S.planes, S.masks, warp, NWARP, cf.C);
             if (tid == 0) {
                 const int rew = S.ctl[2];
                 sum += rew;
@@ -1294,6 +1298,412 @@ rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
     for (int p = tid; p < HW; p += 32 * NWARP)
         dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
     if (tid == 0) {
+        tsteps[env] = t;
+        if (rew_sum)
+            rew_sum[env] = sum;
+        if (S.ctl[3])
+            atomicOr(status + 1, kWarnAction);
+    }
+}
+
+// ============================================================ one warp per environment
+// Boards of at most 16 plane words and at most 16 rules.  A CTA holds
+// blockDim.x / 32 environments, one warp each, every one with its own region
+// of shared memory (FastLayout).  Planes: 0..C-1 tile channels, C the force of
+// the current step, C+1..C+5 the force of actions 0..4 (rebuilt only when the
+// board changes), C+6 all ones; the next step's force is copied into plane C
+// at the end of each step.  Each lane keeps the first four present terms of
+// every rule in registers (EnvRule; a rule with fewer reads the all-ones plane
+// in their place), so a step in which no rule survives them is RPW x 4 shared
+// loads, one vote and the force copy: no barrier, no shared counter.  Rules
+// that do survive continue, one at a time, in a single inlined loop over the
+// remaining terms (four per vote, the next four fetched ahead).  A step with a
+// match combines the SET / CLEAR planes, tests the goal, resets when due and
+// rebuilds the five force planes, all within the warp.
+
+// Per-lane register data of one rule: its valid anchors in this lane's words
+// and the shared addresses and shifts of its first four present terms.
+constexpr int kRegTerms = 4;
+template <int NA>
+struct EnvRule {
+    uint32_t vm[NA];
+    uint32_t a[kRegTerms], s[kRegTerms];
+};
+
+// Anchors of this lane's word u that pass the register-resident terms.
+template <int NA>
+__device__ __forceinline__ uint32_t env_reg_terms(const EnvRule<NA> &f, int u)
+{
+    const uint2 w0 = lds2(f.a[0] + 64 * u), w1 = lds2(f.a[1] + 64 * u);
+    const uint2 w2 = lds2(f.a[2] + 64 * u), w3 = lds2(f.a[3] + 64 * u);
+    const uint32_t x = f.vm[u] & __funnelshift_r(w0.x, w0.y, f.s[0]) & __funnelshift_r(w1.x, w1.y, f.s[1]);
+    return x & __funnelshift_r(w2.x, w2.y, f.s[2]) & __funnelshift_r(w3.x, w3.y, f.s[3]);
+}
+
+// The terms of rule r after its register-resident ones, for one environment,
+// then the rule's write.  `m` holds the anchors live after the register terms;
+// `pbase` is the shared address of this lane's word in plane 0; `pass` a byte
+// offset of an all-zero plane.  Every remaining term is evaluated, eight per
+// iteration with the next eight descriptors already loaded: a rule that gets
+// this far usually has few live anchors, and a warp vote per few terms costs
+// more than the terms it would skip.  Returns (this lane's reward, 1 if this
+// lane matched).
+template <int NA, bool SM>
+__device__ __forceinline__ int2 env_rule_rest(const DevConfig &cf, const uint32_t *tab, uint32_t pbase,
+                                              uint32_t pass, uint32_t *setp, uint32_t *clrp, int r,
+                                              uint32_t (&m)[NA])
+{
+    constexpr int kBatch = 8;
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
+    const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
+    const uint32_t t0 = min(h0.x, (uint32_t)kRegTerms);
+    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)h1.x * 4 + g;
+    const uint32_t nt = h0.x + h0.y;
+    // a missing term reads an all-zero plane as absent: it passes
+    uint2 dn[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j)
+        dn[j] = t0 + j < nt ? ld2<SM>(tp + 4 * (t0 + j)) : make_uint2(pass, kTermAbsent);
+    for (uint32_t t = t0; t < nt; t += kBatch) {
+        uint2 d[kBatch];
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            d[j] = dn[j];
+            dn[j] = t + kBatch + j < nt ? ld2<SM>(tp + 4 * (t + kBatch + j)) : make_uint2(pass, kTermAbsent);
+        }
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            uint32_t x = m[u];
+#pragma unroll
+            for (int j = 0; j < kBatch; ++j) {
+                const uint2 w = lds2(pbase + d[j].x + 64 * u);
+                const uint32_t neg = (uint32_t)((int32_t)d[j].y >> 31);
+                x &= __funnelshift_r(w.x, w.y, d[j].y) ^ neg;
+            }
+            m[u] = x;
+        }
+    }
+    uint32_t cnt = 0;
+#pragma unroll
+    for (int u = 0; u < NA; ++u)
+        cnt += __popc(m[u]);
+    if (cnt == 0)
+        return make_int2(0, 0);
+    const uint4 *op = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, tab[1])) + (size_t)h1.y * 4 + g;
+    for (uint32_t o = 0; o < h0.z; ++o) {
+        const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            if (!m[u])
+                continue;
+            const int w0 = q + 8 * u + (int)ov.x;
+            const uint32_t lo = m[u] << ov.y;
+            const uint32_t hi = ov.y ? (m[u] >> (32u - ov.y)) : 0u;
+            scatter_bits(setp, ov.z, cf.NW, w0, lo, hi);
+            scatter_bits(clrp, ov.w, cf.NW, w0, lo, hi);
+        }
+    }
+    return make_int2((int)h0.w * (int)cnt, 1);
+}
+
+template <typename CellT, int NA, int RPW, bool SM>
+__global__ void __launch_bounds__(128)
+rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
+                        const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
+                        const CellT *__restrict__ init, int32_t *tsteps, int n_steps, uint64_t seed,
+                        const uint8_t *__restrict__ actions, CellT *obs_traj, int32_t *rew_traj,
+                        uint8_t *done_traj, int32_t *rew_sum, uint32_t *status)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const FastLayout L = fast_layout(cf);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const int env = blockIdx.x * (blockDim.x >> 5) + warp;
+    if (env >= cf.B)
+        return;  // whole warp; the kernel has no block-wide barrier
+    unsigned char *mine = smem + (size_t)warp * L.total;
+    FastSmem S;
+    S.planes = reinterpret_cast<uint2 *>(mine + L.planes);
+    S.setp = reinterpret_cast<uint32_t *>(mine + L.setp);
+    S.clrp = reinterpret_cast<uint32_t *>(mine + L.clrp);
+    S.basep = reinterpret_cast<uint32_t *>(mine + L.basep);
+    S.vm = reinterpret_cast<uint32_t *>(mine + L.vm);
+    S.masks = reinterpret_cast<uint32_t *>(mine + L.masks);
+    S.ctl = reinterpret_cast<int *>(mine + L.ctl);
+    S.acts = mine + L.acts;
+    S.rules = reinterpret_cast<uint32_t *>(mine + L.rules);
+
+    const int HW = cf.HW, NW = cf.NW, NWP = cf.NWP, C = cf.C;
+    const int table = cf.rules_per_env ? env : 0;
+    const uint32_t *tab_g = arena + tab_off[table];
+    const uint32_t *tab = SM ? S.rules : tab_g;
+    const uint32_t plane_bytes = (uint32_t)NWP * 8;
+    const uint32_t pass = (uint32_t)(C + 1) * plane_bytes;  // action 0: no force anywhere
+    const uint32_t ones = (uint32_t)(C + 6) * plane_bytes;  // every bit set
+    uint2 *const slot = S.planes + C * NWP;
+    const uint2 *const fplanes = S.planes + (C + 1) * NWP;
+
+    // ---- stage (this warp's environment only)
+    for (int i = lane; i < (C + 7) * NWP; i += 32)
+        S.planes[i] = i < (C + 6) * NWP ? make_uint2(0u, 0u) : make_uint2(0xffffffffu, 0xffffffffu);
+    for (int i = lane; i < C * NW; i += 32) {
+        S.setp[i] = 0u;
+        S.clrp[i] = 0u;
+    }
+    for (int i = lane; i < kShapes * NW; i += 32)
+        S.vm[i] = __ldg(vm_g + i);
+    for (int i = lane; i < 3 * NW; i += 32)
+        S.masks[i] = __ldg(masks_g + i);
+    if (SM) {
+        const uint32_t n = tab_off[table + 1] - tab_off[table];
+        const uint4 *src = reinterpret_cast<const uint4 *>(tab_g);
+        uint4 *d = reinterpret_cast<uint4 *>(S.rules);
+        for (uint32_t i = lane; i < n / 4; i += 32)
+            d[i] = __ldg(src + i);
+    }
+    if (lane < 16)
+        S.ctl[lane] = 0;
+    for (int k = lane; k < kActChunk; k += 32)  // every slot holds an action in 0..4
+        S.acts[k] = k < n_steps ? (uint8_t)action_at(actions, seed, env, k, S.ctl + 3) : (uint8_t)0;
+    __syncwarp();
+    {
+        const CellT *src = cur + (size_t)env * HW, *isrc = init + (size_t)env * HW;
+        for (int base = 0; base < HW; base += 32) {
+            const int p = base + lane;
+            const uint32_t v = p < HW ? (uint32_t)src[p] : 0u;
+            const uint32_t vi = p < HW ? (uint32_t)isrc[p] : 0u;
+            const int w = p >> 5;
+            for (int c = 0; c < C; ++c) {
+                const uint32_t bits = __ballot_sync(0xffffffffu, (v >> c) & 1u);
+                const uint32_t ibits = __ballot_sync(0xffffffffu, (vi >> c) & 1u);
+                if (lane == 0 && w < NW) {
+                    put_word(S.planes, NWP, c, w, bits);
+                    S.basep[c * NW + w] = ibits;
+                }
+            }
+        }
+    }
+    __syncwarp();
+    force_planes(cf, S.planes, S.masks, 0, 1, C + 1);
+    __syncwarp();
+    if (lane < NW)
+        slot[lane] = fplanes[S.acts[0] * NWP + lane];
+
+    // ---- per-lane register data of every rule
+    EnvRule<NA> fr[RPW];
+    const uint32_t pbase = (uint32_t)__cvta_generic_to_shared(S.planes) + q * 8;
+    {
+        const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+#pragma unroll
+        for (int k = 0; k < RPW; ++k) {
+            EnvRule<NA> &f = fr[k];
+#pragma unroll
+            for (int u = 0; u < NA; ++u)
+                f.vm[u] = 0;
+#pragma unroll
+            for (int j = 0; j < kRegTerms; ++j) {
+                f.a[j] = pbase + ones;
+                f.s[j] = 0;
+            }
+            if (k < cf.R) {
+                const uint4 h0 = ld4<SM>(tab + 4 + 8 * k);
+                const uint4 h1 = ld4<SM>(tab + 8 + 8 * k);
+                const uint32_t *vmr = S.vm + ((h1.z >> (8 * g)) & 0xffu) * NW;
+#pragma unroll
+                for (int u = 0; u < NA; ++u) {
+                    const int a = q + 8 * u;
+                    f.vm[u] = a < NW ? vmr[a] : 0u;
+                }
+#pragma unroll
+                for (int j = 0; j < kRegTerms; ++j)
+                    if ((uint32_t)j < h0.x) {  // present terms lead the rule's term list
+                        const uint2 d = ld2<SM>(terms + (size_t)(h1.x + j) * 4 + g);
+                        f.a[j] = pbase + d.x;
+                        f.s[j] = d.y;
+                    }
+            }
+        }
+    }
+    int t = tsteps[env];
+    int goal_left;
+    {
+        int gl = cf.ch_goal < 0;
+        if (cf.ch_goal >= 0)
+            for (int w = lane; w < NW; w += 32)
+                gl |= S.planes[cf.ch_goal * NWP + w].x != 0u;
+        goal_left = __any_sync(0xffffffffu, gl);
+    }
+    __syncwarp();  // the force of step 0
+    const bool traj = rew_traj != nullptr || done_traj != nullptr;
+
+    int sum = 0;
+    uint32_t m[RPW][NA];  // anchors of each rule live after its register terms
+    // Steps in which no rule survives its register terms: t advances, the next
+    // step's force goes into the slot, nothing else changes.  The loop is kept
+    // free of branches around rarely used code, which cost tens of cycles each
+    // even when not taken.  Returns true when step s has a live rule (its masks
+    // left in m for the general step).
+    auto quiet_steps = [&](int &s, int lim, auto traj_tag) -> bool {
+        constexpr bool TRAJ = decltype(traj_tag)::value;
+        while (s < lim && (!cf.auto_reset || (goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps)))) {
+            const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
+            const uint2 f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
+            uint32_t anyall = 0;
+#pragma unroll
+            for (int k = 0; k < RPW; ++k)
+#pragma unroll
+                for (int u = 0; u < NA; ++u) {
+                    m[k][u] = env_reg_terms(fr[k], u);
+                    anyall |= m[k][u];
+                }
+            if (__any_sync(0xffffffffu, anyall != 0u))
+                return true;  // the general step takes it
+            t += 1;
+            if (TRAJ) {
+                const int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+                if (lane == 0) {
+                    if (rew_traj)
+                        rew_traj[(size_t)s * cf.B + env] = 0;
+                    if (done_traj)
+                        done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
+                }
+                if (obs_traj) {
+                    CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
+                    for (int p = lane; p < HW; p += 32)
+                        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+                }
+            }
+            if (lane < NW)
+                slot[lane] = f_next;  // every read of this step's force is behind the vote
+            __syncwarp();
+            ++s;
+        }
+        return false;
+    };
+    const bool any_traj = traj || obs_traj != nullptr;
+    int refilled = 0;
+    for (int s = 0; s < n_steps;) {
+        // actions [s + 128, s + 256) into the ring slots of steps [s - 128, s),
+        // all read by now
+        if (s > 0 && (s & (kActChunk / 2 - 1)) == 0 && s != refilled) {
+            for (int k = lane; k < kActChunk / 2; k += 32)
+                if (s + kActChunk / 2 + k < n_steps)
+                    S.acts[(s + kActChunk / 2 + k) & (kActChunk - 1)] =
+                        (uint8_t)action_at(actions, seed, env, s + kActChunk / 2 + k, S.ctl + 3);
+            __syncwarp();
+            refilled = s;
+        }
+        const int lim = min(n_steps, ((s / (kActChunk / 2)) + 1) * (kActChunk / 2));
+        const bool live_rule = any_traj ? quiet_steps(s, lim, std::integral_constant<bool, true>())
+                                        : quiet_steps(s, lim, std::integral_constant<bool, false>());
+        if (s >= lim)
+            continue;  // the end, or the next refill
+        if (!live_rule) {  // a reset is due: no register masks yet
+#pragma unroll
+            for (int k = 0; k < RPW; ++k)
+#pragma unroll
+                for (int u = 0; u < NA; ++u)
+                    m[k][u] = env_reg_terms(fr[k], u);
+        }
+
+        // ---- general step s: the rest of every live rule, writes
+        const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
+        uint2 f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
+        uint32_t bits = 0;
+#pragma unroll
+        for (int k = 0; k < RPW; ++k) {
+            uint32_t a = 0;
+#pragma unroll
+            for (int u = 0; u < NA; ++u)
+                a |= m[k][u];
+            bits |= (a != 0u ? 1u : 0u) << k;
+        }
+        int rew = 0, changed = 0;
+        {
+            uint32_t live = __reduce_or_sync(0xffffffffu, bits);
+            int2 acc = make_int2(0, 0);
+            while (live) {
+                const int k = __ffs(live) - 1;
+                live &= live - 1;
+                uint32_t mk[NA];
+#pragma unroll
+                for (int u = 0; u < NA; ++u)
+                    mk[u] = 0;
+#pragma unroll
+                for (int kk = 0; kk < RPW; ++kk)
+                    if (kk == k)
+#pragma unroll
+                        for (int u = 0; u < NA; ++u)
+                            mk[u] = m[kk][u];
+                const int2 o = env_rule_rest<NA, SM>(cf, tab, pbase, pass, S.setp, S.clrp, k, mk);
+                acc.x += o.x;
+                acc.y |= o.y;
+            }
+            rew = __reduce_add_sync(0xffffffffu, acc.x);
+            changed = __any_sync(0xffffffffu, acc.y != 0);
+        }
+
+        t += 1;
+        int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+        if (changed || (done && cf.auto_reset)) {
+            __syncwarp();  // every lane's SET / CLEAR bits
+            // combine: a bit changes where any match asks for it; the goal test
+            // of the new board comes with it
+            int gl = cf.ch_goal < 0;
+            for (int i = lane; i < C * NW; i += 32) {
+                const int c = i / NW, w = i - c * NW;
+                uint32_t d = S.planes[c * NWP + w].x;
+                const uint32_t st = S.setp[i], cl = S.clrp[i];
+                if (st | cl) {
+                    S.setp[i] = 0u;
+                    S.clrp[i] = 0u;
+                    d = (d & ~cl) | (~d & st);
+                    put_word(S.planes, NWP, c, w, d);
+                }
+                if (c == cf.ch_goal)
+                    gl |= d != 0u;
+            }
+            goal_left = __any_sync(0xffffffffu, gl);
+            done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+            if (done && cf.auto_reset) {
+                for (int i = lane; i < C * NW; i += 32) {
+                    const int c = i / NW, w = i - c * NW;
+                    put_word(S.planes, NWP, c, w, S.basep[i]);
+                }
+                t = 0;
+                gl = cf.ch_goal < 0;
+                if (cf.ch_goal >= 0)
+                    for (int w = lane; w < NW; w += 32)
+                        gl |= S.basep[cf.ch_goal * NW + w] != 0u;
+                goal_left = __any_sync(0xffffffffu, gl);
+            }
+            __syncwarp();  // the new board
+            force_planes(cf, S.planes, S.masks, 0, 1, C + 1);
+            __syncwarp();  // its force planes
+            f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
+            sum += rew;
+        }
+        // every read of this step's force is behind the step's last vote
+        if (lane < NW)
+            slot[lane] = f_next;
+        __syncwarp();
+        if (traj && lane == 0) {
+            if (rew_traj)
+                rew_traj[(size_t)s * cf.B + env] = rew;
+            if (done_traj)
+                done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
+        }
+        if (obs_traj) {
+            CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
+            for (int p = lane; p < HW; p += 32)
+                dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+        }
+        ++s;
+    }
+    CellT *dst = cur + (size_t)env * HW;
+    for (int p = lane; p < HW; p += 32)
+        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+    if (lane == 0) {
         tsteps[env] = t;
         if (rew_sum)
             rew_sum[env] = sum;
@@ -1620,13 +2030,29 @@ inline int anchor_slots(int NW)
     return na;
 }
 
-// Paths: cf.path 0 = choose, 1 = block per env, 3 = fast rollout.
-// Rollouts: the fast kernel for boards of at most 16 plane words and <= 64
-// rules unless the block path is forced; expansion: one warp per parent for
-// boards of at most 16 plane words unless the block path is forced.
+// Paths: cf.path 0 = choose, 1 = block per env, 2 = fast rollout (several warps
+// per env), 3 = one warp per env.
+// Rollouts: one warp per environment for boards of at most 16 plane words and
+// at most 16 rules, else the fast kernel for <= 64 rules, else (or when forced)
+// the block kernel.  Expansion: one warp per parent for boards of at most 16
+// plane words unless the block path is forced.
+inline bool use_env_warp_rollout(const DevConfig &cf)
+{
+    return cf.NA <= 2 && cf.R <= 16 && (cf.path == 0 || cf.path == 3);
+}
 inline bool use_fast_rollout(const DevConfig &cf) { return cf.NA <= 2 && cf.R <= 64 && cf.path != 1; }
 inline bool use_warp_expand(const DevConfig &cf) { return cf.NA <= 2 && cf.path != 1; }
 
 constexpr int kDynSmemLimit = 200 * 1024;
+
+// Environments per CTA of the one-warp-per-environment rollout: four, fewer
+// when their shared memory would not fit.
+inline int env_warps_per_cta(const DevConfig &cf)
+{
+    int epb = 4;
+    while (epb > 1 && (size_t)epb * fast_layout(cf).total > (size_t)kDynSmemLimit)
+        epb /= 2;
+    return epb;
+}
 
 }  // namespace av

@@ -213,7 +213,7 @@ def test_dense_matches_stress_apply():
 
 
 # ------------------------------------------------- both kernel paths
-@pytest.mark.parametrize("path", ["block", "fast", "fast8"])
+@pytest.mark.parametrize("path", ["block", "fast", "fast8", "warp"])
 @pytest.mark.parametrize("key,batch,steps", [(1, 3, 60), (2, 9, 70), (3, 7, 230), (4, 4, 30)])
 def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
     monkeypatch.setenv("AV_KERNEL_PATH", path.rstrip("8"))
@@ -233,7 +233,7 @@ def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
     env.close()
 
 
-@pytest.mark.parametrize("path", ["block", "fast", "fast8"])
+@pytest.mark.parametrize("path", ["block", "fast", "fast8", "warp"])
 @pytest.mark.parametrize("H,W,C,shapes,R", [
     (1, 1, 1, ((1, 1),), 2),
     (7, 9, 3, ((3, 3), (5, 5), (1, 4)), 4),
@@ -241,6 +241,8 @@ def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
     (2, 64, 9, ((1, 5), (2, 2)), 3),
     (20, 21, 6, ((3, 3), (2, 4)), 9),  # 420 cells: two anchor words per lane
     (16, 16, 5, ((1, 1), (1, 2)), 40),  # many rules: several per warp
+    (16, 16, 5, ((1, 1), (1, 2)), 16),  # the most rules one warp per environment holds
+    (12, 16, 4, ((2, 2), (1, 3)), 11),
 ])
 def test_both_kernel_paths_edges(monkeypatch, path, H, W, C, shapes, R):
     monkeypatch.setenv("AV_KERNEL_PATH", path.rstrip("8"))
