@@ -239,6 +239,15 @@ void compile_table(const av_rule *rules, const DevConfig &cf, const double *dens
             }
             ++n_terms;
         }
+        // padding: the terms after the first kRegTerms present ones fill whole batches
+        const int after = (int)all.size() - std::min((int)pres.size(), kRegTerms);
+        for (int j = after; j % kRestBatch != 0; ++j) {
+            for (int g = 0; g < 4; ++g) {
+                terms.push_back((uint32_t)((cf.C + 1) * cf.NWP * 8));
+                terms.push_back(kTermAbsent);
+            }
+            ++n_terms;
+        }
         uint32_t no = 0;
         for (int i0 = 0; i0 < p.h; ++i0)
             for (int k0 = 0; k0 < p.w; ++k0) {

@@ -29,7 +29,9 @@
 //                        (h'-1)*5 + (w'-1)), 0
 //   terms   (uint2, 16-byte aligned, [term][rotation]):
 //           (byte offset of plane entry c*NWP + (s >> 5), s & 31 | kTermAbsent
-//           for an absent term; funnel shifts use only the low five bits)
+//           for an absent term; funnel shifts use only the low five bits);
+//           each rule's list is followed by padding terms up to a whole
+//           number of kRestBatch terms after its first kRegTerms present ones
 //   outputs (uint4, [output][rotation]): (s >> 5, s & 31, set bits, clear bits)
 #pragma once
 
@@ -50,6 +52,13 @@ constexpr int kMaxSmemRuleWords = 8192;  // stage a rule table in shared memory 
 constexpr uint32_t kStatusVisitedOverflow = 1u;
 constexpr uint32_t kWarnAction = 1u;
 constexpr uint32_t kTermAbsent = 0x80000000u;  // flag in a term's shift word
+// One warp per environment: present terms of a rule held in registers, and the
+// batch in which the remaining terms are evaluated.  Each rule's term list is
+// padded so that the terms after the register ones fill whole batches; a
+// padding term reads plane C + 1 (the force of action 0, zero everywhere in
+// that kernel's layout) as absent, so it passes.
+constexpr int kRegTerms = 4;
+constexpr int kRestBatch = 4;
 
 struct DevConfig {
     int B, H, W, C, HW, NW, NWP, NA;  // NW plane words; NWP doubled entries per plane; NA words per lane
@@ -1323,7 +1332,6 @@ rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
 
 // Per-lane register data of one rule: its valid anchors in this lane's words
 // and the shared addresses and shifts of its first four present terms.
-constexpr int kRegTerms = 4;
 template <int NA>
 struct EnvRule {
     uint32_t vm[NA];
@@ -1334,54 +1342,64 @@ struct EnvRule {
 template <int NA>
 __device__ __forceinline__ uint32_t env_reg_terms(const EnvRule<NA> &f, int u)
 {
-    const uint2 w0 = lds2(f.a[0] + 64 * u), w1 = lds2(f.a[1] + 64 * u);
-    const uint2 w2 = lds2(f.a[2] + 64 * u), w3 = lds2(f.a[3] + 64 * u);
-    const uint32_t x = f.vm[u] & __funnelshift_r(w0.x, w0.y, f.s[0]) & __funnelshift_r(w1.x, w1.y, f.s[1]);
-    return x & __funnelshift_r(w2.x, w2.y, f.s[2]) & __funnelshift_r(w3.x, w3.y, f.s[3]);
+    uint32_t x = f.vm[u];
+#pragma unroll
+    for (int j = 0; j < kRegTerms; ++j) {
+        const uint2 w = lds2(f.a[j] + 64 * u);
+        x &= __funnelshift_r(w.x, w.y, f.s[j]);
+    }
+    return x;
 }
 
 // The terms of rule r after its register-resident ones, for one environment,
 // then the rule's write.  `m` holds the anchors live after the register terms;
-// `pbase` is the shared address of this lane's word in plane 0; `pass` a byte
-// offset of an all-zero plane.  Every remaining term is evaluated, eight per
-// iteration with the next eight descriptors already loaded: a rule that gets
-// this far usually has few live anchors, and a warp vote per few terms costs
-// more than the terms it would skip.  Returns (this lane's reward, 1 if this
-// lane matched).
+// `pbase` is the shared address of this lane's word in plane 0.  Every
+// remaining term is evaluated, kRestBatch per iteration (the padded list has
+// whole batches) with the next batch's descriptors already loaded: a rule that
+// gets this far usually has few live anchors, and a warp vote per few terms
+// costs more than the terms it would skip.  Returns (this lane's reward, 1 if
+// this lane matched).
 template <int NA, bool SM>
 __device__ __forceinline__ int2 env_rule_rest(const DevConfig &cf, const uint32_t *tab, uint32_t pbase,
-                                              uint32_t pass, uint32_t *setp, uint32_t *clrp, int r,
-                                              uint32_t (&m)[NA])
+                                              uint32_t *setp, uint32_t *clrp, int r, uint32_t (&m)[NA])
 {
-    constexpr int kBatch = 8;
     const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
     const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
     const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
     const uint32_t t0 = min(h0.x, (uint32_t)kRegTerms);
-    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)h1.x * 4 + g;
-    const uint32_t nt = h0.x + h0.y;
-    // a missing term reads an all-zero plane as absent: it passes
-    uint2 dn[kBatch];
+    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)(h1.x + t0) * 4 + g;
+    const uint32_t nb = (h0.x + h0.y - t0 + kRestBatch - 1) / kRestBatch;  // padded batches
+    uint2 dn[kRestBatch];
+    if (nb > 0) {
 #pragma unroll
-    for (int j = 0; j < kBatch; ++j)
-        dn[j] = t0 + j < nt ? ld2<SM>(tp + 4 * (t0 + j)) : make_uint2(pass, kTermAbsent);
-    for (uint32_t t = t0; t < nt; t += kBatch) {
-        uint2 d[kBatch];
+        for (int j = 0; j < kRestBatch; ++j)
+            dn[j] = ld2<SM>(tp + 4 * j);
+    }
+    for (uint32_t b = 0; b < nb; ++b) {
+        uint2 d[kRestBatch];
 #pragma unroll
-        for (int j = 0; j < kBatch; ++j) {
+        for (int j = 0; j < kRestBatch; ++j)
             d[j] = dn[j];
-            dn[j] = t + kBatch + j < nt ? ld2<SM>(tp + 4 * (t + kBatch + j)) : make_uint2(pass, kTermAbsent);
+        if (b + 1 < nb) {
+            tp += 4 * kRestBatch;
+#pragma unroll
+            for (int j = 0; j < kRestBatch; ++j)
+                dn[j] = ld2<SM>(tp + 4 * j);
         }
 #pragma unroll
         for (int u = 0; u < NA; ++u) {
-            uint32_t x = m[u];
+            uint32_t v[kRestBatch];
 #pragma unroll
-            for (int j = 0; j < kBatch; ++j) {
+            for (int j = 0; j < kRestBatch; ++j) {
                 const uint2 w = lds2(pbase + d[j].x + 64 * u);
-                const uint32_t neg = (uint32_t)((int32_t)d[j].y >> 31);
-                x &= __funnelshift_r(w.x, w.y, d[j].y) ^ neg;
+                v[j] = __funnelshift_r(w.x, w.y, d[j].y) ^ (uint32_t)((int32_t)d[j].y >> 31);
             }
-            m[u] = x;
+            // a balanced AND: the terms of a batch do not wait on one another
+            uint32_t x = v[0];
+#pragma unroll
+            for (int j = 1; j < kRestBatch; ++j)
+                x &= v[j];
+            m[u] &= x;
         }
     }
     uint32_t cnt = 0;
@@ -1438,7 +1456,6 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
     const uint32_t *tab_g = arena + tab_off[table];
     const uint32_t *tab = SM ? S.rules : tab_g;
     const uint32_t plane_bytes = (uint32_t)NWP * 8;
-    const uint32_t pass = (uint32_t)(C + 1) * plane_bytes;  // action 0: no force anywhere
     const uint32_t ones = (uint32_t)(C + 6) * plane_bytes;  // every bit set
     uint2 *const slot = S.planes + C * NWP;
     const uint2 *const fplanes = S.planes + (C + 1) * NWP;
@@ -1635,7 +1652,7 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
 #pragma unroll
                         for (int u = 0; u < NA; ++u)
                             mk[u] = m[kk][u];
-                const int2 o = env_rule_rest<NA, SM>(cf, tab, pbase, pass, S.setp, S.clrp, k, mk);
+                const int2 o = env_rule_rest<NA, SM>(cf, tab, pbase, S.setp, S.clrp, k, mk);
                 acc.x += o.x;
                 acc.y |= o.y;
             }
