@@ -36,7 +36,9 @@ import workload as wk  # noqa: E402
 
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 KERNEL_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "kernels.cuh")
-PROFILE = os.path.join(ROOT, "profiles", "rollout_kernel_grid16_b1024.md")
+PROFILE_DIR = os.path.join(ROOT, "profiles")
+# rollout kernel launched for each av_rollout_path value
+KERNEL_NAMES = {1: "rollout_kernel", 2: "rollout_fast_kernel", 3: "rollout_env_warp_kernel"}
 SM_COUNT_GB300 = 152
 # 32-bit integer instructions issued per SM per clock: 4 schedulers x 32 lanes.
 # The committed probe (--int-probe) reaches 113-114 of them for IADD3, SHF and
@@ -80,33 +82,68 @@ def algorithmic_ops(wl: wk.Workload, rules: np.ndarray) -> float:
 
 # --------------------------------------------------------------- clocks
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi samples every 25 ms; stats over those taken inside the timed
+    window (between mark_start and mark_end)."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index: int):
         self.index = index
         self.proc = None
+        self.rows = []
+        self.t0 = self.t1 = None
 
-    def start(self):
+    def start(self, wait_s: float = 5.0):
+        import threading
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "25"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
+            return
+
+        def reader():
+            for line in self.proc.stdout:
+                r = [x.strip() for x in line.split(",")]
+                if len(r) >= 9:
+                    self.rows.append((self._when(r[0]), r))
+
+        threading.Thread(target=reader, daemon=True).start()
+        end = time.time() + wait_s
+        while not self.rows and time.time() < end:  # sampling has begun
+            time.sleep(0.01)
+
+    @staticmethod
+    def _when(stamp: str) -> float | None:
+        import datetime
+        try:
+            return datetime.datetime.strptime(stamp, "%Y/%m/%d %H:%M:%S.%f").timestamp()
+        except ValueError:
+            return None
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+        end = self.t1 + 0.2
+        while time.time() < end and not any(t and t >= self.t1 for t, _ in self.rows[-3:]):
+            time.sleep(0.01)
 
     def stop(self) -> dict | None:
         if self.proc is None:
             return None
         self.proc.terminate()
         try:
-            out, _ = self.proc.communicate(timeout=5)
+            self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
-            out, _ = self.proc.communicate()
-        rows = [r.split(",") for r in out.strip().splitlines() if r.count(",") >= 8]
+        inside = [r for t, r in self.rows if t is not None and self.t0 is not None
+                  and self.t0 <= t <= self.t1]
+        rows = inside or [r for _, r in self.rows]
         if not rows:
             return None
         mhz = [float(r[1]) for r in rows]
@@ -118,10 +155,19 @@ class ClockSampler:
                 if r[col].strip().lower() == "active":
                     reasons.add(name)
         return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows)}
+                "samples": len(rows), "samples_in_timed_region": len(inside),
+                "power_w_max": max(float(r[3]) for r in rows)}
 
 
-# -------------------------------------------------------------- helpers
+def valid_anchor_rules(wl: wk.Workload, rules: np.ndarray) -> float:
+    """Valid (anchor, rule rotation) pairs per env-step, averaged over envs."""
+    h = rules["h"].astype(np.int64)
+    w = rules["w"].astype(np.int64)
+    va = np.clip(wl.H - h + 1, 0, None) * np.clip(wl.W - w + 1, 0, None)
+    vb = np.clip(wl.H - w + 1, 0, None) * np.clip(wl.W - h + 1, 0, None)
+    return float((2 * va + 2 * vb).sum(-1).mean())
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -136,11 +182,15 @@ def measured_peaks() -> dict:
         return {}
 
 
-def profile_traffic() -> float | None:
-    """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source."""
+def profile_path(kernel: str, wl) -> str:
+    return os.path.join(PROFILE_DIR, f"{kernel}_{wl.name}.md")
+
+
+def profile_traffic(kernel: str, wl) -> float | None:
+    """DRAM bytes per launch from the committed ncu summary of this kernel on
+    this workload, if it was taken on the current kernel source."""
     try:
-        text = open(PROFILE).read()
+        text = open(profile_path(kernel, wl)).read()
     except OSError:
         return None
     m = re.search(r"kernel_source_sha256:\s*([0-9a-f]{16,64})", text)
@@ -273,6 +323,7 @@ def run_ours(args, wl):
     sampler = ClockSampler(torch.cuda.current_device() if world == 1 else local)
     sampler.start()
     barrier()
+    sampler.mark_start()
     t_wall = time.perf_counter()
     for i in range(args.steps):
         flush.fill_(i & 0xff)  # evict L2 between timed launches (outside the events)
@@ -281,6 +332,7 @@ def run_ours(args, wl):
         ends[i].record(stream)
     barrier()
     wall = time.perf_counter() - t_wall
+    sampler.mark_end()
     clocks = sampler.stop()
     env.sync()
     ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
@@ -293,7 +345,6 @@ def run_ours(args, wl):
         total_ms = float(tt.item())
     env_steps = wl.batch * wl.steps * args.steps * world
     value = env_steps / (total_ms / 1e3)
-    cells_rules = wl.H * wl.W * wl.n_rules * 4
 
     # ---- e2e: the same launch through host buffers (pinned), copies timed
     host_in = g0.cpu().pin_memory()
@@ -325,21 +376,27 @@ def run_ours(args, wl):
         peak_ops = SM_COUNT_GB300 * INT_LANES_PER_SM * sm_max * 1e6 / 1e9  # Gop/s
         ops = algorithmic_ops(wl, rules)
         achieved = ops * wl.batch * wl.steps / (kernel_ms / 1e3) / 1e9
-        traffic = profile_traffic()
+        kernel = KERNEL_NAMES[av.av_rollout_path(env.h)]
+        traffic = profile_traffic(kernel, wl)
         line = {
             "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
             "data": "synthetic", "config": config_dict(wl),
-            "cell_rule_updates_per_s": value * cells_rules,
+            "cell_rule_updates_per_s": value * wl.H * wl.W * wl.n_rules * 4,
+            "valid_anchor_rule_tests_per_s": value * valid_anchor_rules(wl, rules),
             "e2e": {"value": e2e_value, "unit": "env-steps/s",
                     "h2d_bytes_per_step": int(host_in.numel() * host_in.element_size()),
                     "d2h_bytes_per_step": int(host_out.numel() * host_out.element_size())},
             "roofline": {"bound": "alu", "achieved": achieved, "peak": peak_ops,
                          "unit": "Gop/s", "frac": achieved / peak_ops,
                          "traffic": traffic,
-                         "kernel": "rollout_kernel<uint8_t>",
+                         "kernel": kernel,
                          "ops_per_env_step": ops,
+                         "ops_basis": "full evaluation: every term and output entry of every"
+                                      " rule rotation at every valid anchor, one 32-bit word"
+                                      " op per 32 anchors; the kernels stop evaluating a rule"
+                                      " once no anchor is live, so frac can exceed 1",
                          "peak_from": f"{SM_COUNT_GB300} SMs x {INT_LANES_PER_SM} int32 lanes/clk"
                                       f" x {sm_max:.0f} MHz (sm_max_mhz of measured peaks)"},
             "gpu_launches": args.steps,
@@ -373,7 +430,7 @@ def run_int_probe() -> int:
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--config", type=int, default=2, choices=(2, 3, 5))

@@ -225,6 +225,17 @@ int av_sync(av_handle *h);
 /* Warning bits seen since the last call (synchronises); see AV_WARN_*. */
 int av_warnings(av_handle *h, uint32_t *bits);
 
+/* Which rollout kernel av_step / av_rollout launch for this handle:
+ * AV_PATH_BLOCK (one CTA per environment), AV_PATH_FAST (several warps per
+ * environment, boards of at most 512 cells and at most 64 rules) or
+ * AV_PATH_WARP (one warp per environment, boards of at most 512 cells and at
+ * most 16 rules).  The library picks the last that fits; the environment
+ * variable AV_KERNEL_PATH=block|fast|warp, read by av_create, forces one for
+ * tests and measurements.  Writes the path to *path; AV_EINVAL for a null
+ * argument.  No GPU work. */
+enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3 };
+int av_rollout_path(av_handle *h, int32_t *path);
+
 /* Static description of a status code. */
 const char *av_strerror(int status);
 

@@ -20,10 +20,11 @@ LIB_PATH = os.path.join(_PKG, "libautoverse.so")
 
 AV_OK, AV_EINVAL, AV_ENOMEM, AV_ECUDA, AV_ESTATE, AV_EDEVICE = 0, -1, -2, -3, -4, -5
 AV_WARN_ACTION = 1
+AV_PATH_BLOCK, AV_PATH_FAST, AV_PATH_WARP = 1, 2, 3
 RULE_BYTES = 408
 EXPORTS = ("av_create", "av_destroy", "av_reset", "av_set_state", "av_get_state", "av_step",
            "av_rollout", "av_expand", "av_search_init", "av_select", "av_select_static", "av_sync",
-           "av_warnings", "av_strerror", "av_last_error")
+           "av_warnings", "av_rollout_path", "av_strerror", "av_last_error")
 AV_SELECT_STATIC_MAX_HASHES = 1 << 21
 
 
@@ -72,6 +73,7 @@ def load() -> ctypes.CDLL:
                              vp, vp, vp, vp, i32, vp, up],
         "av_sync": [vp],
         "av_warnings": [vp, ctypes.POINTER(ctypes.c_uint32)],
+        "av_rollout_path": [vp, ctypes.POINTER(ctypes.c_int32)],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -215,6 +217,12 @@ def av_warnings(h) -> int:
     bits = ctypes.c_uint32()
     _check(h, "av_warnings", load().av_warnings(h, ctypes.byref(bits)))
     return int(bits.value)
+
+
+def av_rollout_path(h) -> int:
+    path = ctypes.c_int32()
+    _check(h, "av_rollout_path", load().av_rollout_path(h, ctypes.byref(path)))
+    return int(path.value)
 
 
 class Env:

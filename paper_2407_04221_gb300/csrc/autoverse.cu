@@ -733,6 +733,14 @@ int av_sync(av_handle *h)
     return AV_OK;
 }
 
+int av_rollout_path(av_handle *h, int32_t *path)
+{
+    if (!h || !path)
+        return AV_EINVAL;
+    *path = use_env_warp_rollout(h->cf) ? AV_PATH_WARP : use_fast_rollout(h->cf) ? AV_PATH_FAST : AV_PATH_BLOCK;
+    return AV_OK;
+}
+
 int av_warnings(av_handle *h, uint32_t *bits)
 {
     if (!h || !bits)

@@ -213,14 +213,18 @@ def test_dense_matches_stress_apply():
 
 
 # ------------------------------------------------- both kernel paths
+_PATH_IDS = {"block": 1, "fast": 2, "fast8": 2, "warp": 3}
+
 @pytest.mark.parametrize("path", ["block", "fast", "fast8", "warp"])
 @pytest.mark.parametrize("key,batch,steps", [(1, 3, 60), (2, 9, 70), (3, 7, 230), (4, 4, 30)])
 def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
+    import paper_2407_04221_gb300 as av
     monkeypatch.setenv("AV_KERNEL_PATH", path.rstrip("8"))
     if path.endswith("8"):
         monkeypatch.setenv("AV_FAST_WARPS", "8")
     wl = wk.WORKLOADS[key].scaled(batch=batch)
     env, cfg, rules, cum = make(wl, 11 + key)
+    assert av.av_rollout_path(env.h) == _PATH_IDS[path]
     s = wk.seeds(11 + key)
     g0 = to_np(env.reset(s["reset"]))
     res = env.rollout(steps, s["actions"], trajectory=True)
@@ -245,6 +249,7 @@ def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
     (12, 16, 4, ((2, 2), (1, 3)), 11),
 ])
 def test_both_kernel_paths_edges(monkeypatch, path, H, W, C, shapes, R):
+    import paper_2407_04221_gb300 as av
     monkeypatch.setenv("AV_KERNEL_PATH", path.rstrip("8"))
     if path.endswith("8"):
         monkeypatch.setenv("AV_FAST_WARPS", "8")
@@ -255,6 +260,9 @@ def test_both_kernel_paths_edges(monkeypatch, path, H, W, C, shapes, R):
     if C > 2:
         g0[:, H // 2, W // 2] |= 1 << 2
     env, cfg, _, _ = make(wl, 0, rules=rules, cum=None)
+    # one warp per environment holds at most 16 rules; beyond that the fast kernel runs
+    want = av.AV_PATH_FAST if path == "warp" and R > 16 else _PATH_IDS[path]
+    assert av.av_rollout_path(env.h) == want
     env.set_state(to_dev(g0), set_as_init=True)
     res = env.rollout(15, 123, trajectory=True)
     ref = oracle.rollout(cfg, rules, g0, g0, np.zeros(5), 15, 123, trajectory=True)
