@@ -229,10 +229,12 @@ int av_warnings(av_handle *h, uint32_t *bits);
  * AV_PATH_BLOCK (one CTA per environment), AV_PATH_FAST (several warps per
  * environment, boards of at most 512 cells and at most 64 rules) or
  * AV_PATH_WARP (one warp per environment, boards of at most 512 cells and at
- * most 16 rules).  The library picks the last that fits; the environment
- * variable AV_KERNEL_PATH=block|fast|warp, read by av_create, forces one for
- * tests and measurements.  Writes the path to *path; AV_EINVAL for a null
- * argument.  No GPU work. */
+ * most 16 rules).  The library picks the last that fits, except that rule sets
+ * expected to keep matching on most steps (estimated by av_create from the
+ * rules' leading present terms and the init_cum densities) take the block
+ * kernel.  The environment variable AV_KERNEL_PATH=block|fast|warp, read by
+ * av_create, forces one for tests and measurements.  Writes the path to
+ * *path; AV_EINVAL for a null argument.  No GPU work. */
 enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3 };
 int av_rollout_path(av_handle *h, int32_t *path);
 

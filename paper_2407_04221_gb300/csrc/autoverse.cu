@@ -154,8 +154,10 @@ void turn_position(int h, int w, int g, int &i, int &k)
 // channel almost always holds), the most common channels first.  `density`
 // (C entries, or null) is each tile channel's share of cells in the initial
 // maps; without it every tile channel counts as equally common.
-void compile_table(const av_rule *rules, const DevConfig &cf, const double *density, std::vector<uint32_t> &arena)
+void compile_table(const av_rule *rules, const DevConfig &cf, const double *density, std::vector<uint32_t> &arena,
+                   double *live_rules)
 {
+    *live_rules = 0.0;
     const size_t base = arena.size();
     const int R = cf.R;
     std::vector<uint32_t> hdr(8 * (size_t)R, 0), terms, outs;
@@ -215,7 +217,28 @@ void compile_table(const av_rule *rules, const DevConfig &cf, const double *dens
                     found = 1;
                 }
             }
-    uint32_t *hd = &hdr[8 * (size_t)r];
+        // Expected anchors per step that pass the rule's first kRegTerms
+        // present terms, channels taken as independent with the densities above
+        // (an exclusive pair passes nowhere), capped at one: the expected chance
+        // that the rule needs more than its register-resident terms in a step.
+        {
+            double pass = 1.0;
+            const size_t nreg = std::min(pres.size(), (size_t)kRegTerms);
+            const bool exclusive = nreg >= 2 && pres[0].i == pres[1].i && pres[0].k == pres[1].k &&
+                                   pres[0].c < cf.C && pres[1].c < cf.C && pres[0].c != cf.ch_player &&
+                                   pres[1].c != cf.ch_player;
+            for (size_t j = 0; j < nreg; ++j)
+                pass *= pres[j].dens;
+            if (exclusive)
+                pass = 0.0;
+            double anchors = 0.0;
+            for (int g = 0; g < 4; ++g) {
+                const int hh = (g & 1) ? p.w : p.h, ww = (g & 1) ? p.h : p.w;
+                anchors += (double)std::max(0, cf.H - hh + 1) * std::max(0, cf.W - ww + 1);
+            }
+            *live_rules += std::min(1.0, anchors * pass);
+        }
+        uint32_t *hd = &hdr[8 * (size_t)r];
         hd[0] = (uint32_t)pres.size();
         hd[1] = (uint32_t)absn.size();
         hd[3] = (uint32_t)p.reward;
@@ -422,6 +445,7 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
 
     std::vector<uint32_t> arena, tab_off((size_t)n_tables + 1);
     uint32_t max_words = 0;
+    double live_sum = 0.0;  // expected rules per step that pass their register terms, summed over tables
     // tile-channel densities of the initial maps, per table, for the term order
     std::vector<double> density;
     if (cfg->init_cum) {
@@ -447,10 +471,18 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
         const double *dens = nullptr;
         if (!density.empty())
             dens = density.data() + (density.size() > (size_t)cf.C && n_tables == cf.B ? (size_t)t * cf.C : 0);
-        compile_table(rules + (size_t)t * cfg->n_rules, cf, dens, arena);
+        double live = 0.0;
+        compile_table(rules + (size_t)t * cfg->n_rules, cf, dens, arena, &live);
+        live_sum += live;
         max_words = std::max(max_words, (uint32_t)arena.size() - tab_off[t]);
     }
     tab_off[n_tables] = (uint32_t)arena.size();
+    // Environments whose rules keep passing their register-resident terms step
+    // after step do most of their work in the one-warp kernel's general step,
+    // one rule after another; the block kernel spreads the rules over eight
+    // warps.  Busy when, on average, an environment expects half a rule or
+    // more per step to get past its register terms.
+    cf.busy = live_sum / n_tables >= 0.5 ? 1 : 0;
     cf.rule_words = max_words <= (uint32_t)kMaxSmemRuleWords ? (int)max_words : 0;
     std::vector<uint32_t> vm = valid_masks(cf);
     std::vector<uint32_t> masks = column_masks(cf);

@@ -67,6 +67,7 @@ struct DevConfig {
     int cell_bytes;
     int rule_words;  // largest rule table (words) when tables are staged in shared memory, else 0
     int path;        // 0: choose; 1: block kernels; 2: fast rollout; 3: one warp per env
+    int busy;        // rules expected to pass their register terms on most steps (host estimate)
     int fast_warps;  // fast rollout: warps per environment (4, or 8 when set to 8)
 };
 
@@ -2051,13 +2052,16 @@ inline int anchor_slots(int NW)
 // per env), 3 = one warp per env.
 // Rollouts: one warp per environment for boards of at most 16 plane words and
 // at most 16 rules, else the fast kernel for <= 64 rules, else (or when forced)
-// the block kernel.  Expansion: one warp per parent for boards of at most 16
+// the block kernel; rule sets flagged busy take the block kernel.  Expansion: one warp per parent for boards of at most 16
 // plane words unless the block path is forced.
 inline bool use_env_warp_rollout(const DevConfig &cf)
 {
-    return cf.NA <= 2 && cf.R <= 16 && (cf.path == 0 || cf.path == 3);
+    return cf.NA <= 2 && cf.R <= 16 && ((cf.path == 0 && !cf.busy) || cf.path == 3);
 }
-inline bool use_fast_rollout(const DevConfig &cf) { return cf.NA <= 2 && cf.R <= 64 && cf.path != 1; }
+inline bool use_fast_rollout(const DevConfig &cf)
+{
+    return cf.NA <= 2 && cf.R <= 64 && ((cf.path == 0 && !cf.busy) || cf.path == 2 || cf.path == 3);
+}
 inline bool use_warp_expand(const DevConfig &cf) { return cf.NA <= 2 && cf.path != 1; }
 
 constexpr int kDynSmemLimit = 200 * 1024;
