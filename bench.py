@@ -416,6 +416,243 @@ def run_ours(args, wl):
     return 0
 
 
+# ------------------------------------------------------------ search (config 4)
+def search_ops_per_child(wl, rules) -> float:
+    """Full-evaluation ops of one child's step plus its FNV-1a-64 hash: per
+    board byte one 64-bit xor and one 64-bit multiply, counted as 2 + 4
+    32-bit operations."""
+    return algorithmic_ops(wl, rules) + 6.0 * wl.H * wl.W * wl.cell_bytes
+
+
+def search_children(trace_n) -> int:
+    """Children generated by one search: 5 per parent expanded.  The root is
+    the only parent of iteration 0; later iterations expand the frontier the
+    previous one selected."""
+    import torch
+    n = trace_n.to(torch.int64)
+    parents = n.shape[0] + int(n[:, :-1].sum())
+    return 5 * parents
+
+
+def run_search(args, wl):
+    """One benchmark step = one full search per env (Env.search: iterations of
+    av_expand + av_select from the reset boards); env-steps count children."""
+    import torch
+
+    import paper_2407_04221_gb300 as av
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    seed = args.seed + 1000 * rank
+    _, rules, cum = wk.make(wl, seed)
+    fields = wk.config_fields(wl)
+    k, iters = wl.frontier, wl.iterations
+    env = av.Env(fields, rules, cum, device=dev, search_capacity=1 + k * iters)
+    s = wk.seeds(seed)
+    roots = env.reset(s["reset"]).clone()
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        res = env.search(roots, iters, k)
+    torch.cuda.synchronize(dev)
+    env.sync()
+    children = search_children(res["trace_n"])  # the same every step: same roots, same rules
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(torch.cuda.current_device() if world == 1 else local)
+    sampler.start()
+    barrier()
+    sampler.mark_start()
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.fill_(i & 0xff)
+        starts[i].record(stream)
+        env.search(roots, iters, k)
+        ends[i].record(stream)
+    barrier()
+    wall = time.perf_counter() - t_wall
+    sampler.mark_end()
+    clocks = sampler.stop()
+    env.sync()
+    total_ms = sum(a.elapsed_time(b) for a, b in zip(starts, ends))
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    value = children * args.steps * world / (total_ms / 1e3)
+
+    # ---- the expand kernel alone: events around each av_expand of one search
+    # (the same calls, in the same order, as Env.search)
+    i32, u8 = torch.int32, torch.uint8
+    front, nxt = env.boards(wl.batch, k), env.boards(wl.batch, k)
+    cum_, ncum = (torch.zeros(wl.batch, k, dtype=i32, device=dev) for _ in range(2))
+    hsh, nhsh = (torch.zeros(wl.batch, k, dtype=torch.int64, device=dev) for _ in range(2))
+    live, nlive = (torch.zeros(wl.batch, k, dtype=u8, device=dev) for _ in range(2))
+    n = torch.ones(wl.batch, dtype=i32, device=dev)
+    nn = torch.zeros_like(n)
+    front[:, 0].copy_(roots)
+    rh = torch.zeros(wl.batch, dtype=torch.int64, device=dev)
+    rl = torch.zeros(wl.batch, dtype=u8, device=dev)
+    av.av_search_init(env.h, roots, rh, rl)
+    hsh[:, 0].copy_(rh)
+    live[:, 0].copy_(rl)
+    ch = env.boards(wl.batch, k, 5)
+    rw = torch.zeros(wl.batch, k, 5, dtype=i32, device=dev)
+    dn = torch.zeros(wl.batch, k, 5, dtype=u8, device=dev)
+    chh = torch.zeros(wl.batch, k, 5, dtype=torch.int64, device=dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(iters)]
+    parents = []
+    for it in range(iters):
+        parents.append(n.clone())
+        ev[it][0].record(stream)
+        av.av_expand(env.h, front, k, ch, rw, dn, chh, n)
+        ev[it][1].record(stream)
+        av.av_select(env.h, k, n, cum_, live, ch, rw, dn, chh, k, nxt, ncum, nhsh, nlive, nn)
+        front, nxt, cum_, ncum, hsh, nhsh = nxt, front, ncum, cum_, nhsh, hsh
+        live, nlive, n, nn = nlive, live, nn, n
+    torch.cuda.synchronize(dev)
+    env.sync()
+    exp_ms = sum(a.elapsed_time(b) for a, b in ev)
+    exp_children = 5 * int(sum(int(p.sum()) for p in parents))
+
+    # ---- e2e: roots from pinned host memory, best cumulative reward back
+    host_roots = roots.cpu().pin_memory()
+    host_best = torch.empty(wl.batch, iters, dtype=torch.int32).pin_memory()
+    dev_roots = torch.empty_like(roots)
+    e2e_steps = max(3, min(args.steps, 10))
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        dev_roots.copy_(host_roots, non_blocking=True)
+        r = env.search(dev_roots, iters, k)
+        host_best.copy_(r["trace_best"], non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    e2e_value = children * world / (e2e_ms / 1e3)
+
+    if rank == 0:
+        peaks = measured_peaks()
+        sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+        peak_ops = SM_COUNT_GB300 * INT_LANES_PER_SM * sm_max * 1e6 / 1e9
+        ops = search_ops_per_child(wl, rules)
+        achieved = ops * exp_children / (exp_ms / 1e3) / 1e9
+        kernel = "expand_warp_kernel" if wl.H * wl.W <= 512 else "expand_kernel"
+        line = {
+            "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+            "data": "synthetic",
+            "config": dict(config_dict(wl), frontier=k, iterations=iters,
+                           children_per_step=children,
+                           rules_note="rules 0-1 of every table are the maze game's move and"
+                                      " eat rules, the rest random"),
+            "e2e": {"value": e2e_value, "unit": "env-steps/s",
+                    "h2d_bytes_per_step": int(host_roots.numel() * host_roots.element_size()),
+                    "d2h_bytes_per_step": int(host_best.numel() * host_best.element_size())},
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": peak_ops,
+                         "unit": "Gop/s", "frac": achieved / peak_ops,
+                         "traffic": profile_traffic(kernel, wl), "kernel": kernel,
+                         "ops_per_child": ops,
+                         "ops_basis": "full evaluation of the child's step (as for rollouts)"
+                                      " plus FNV-1a-64 over the child's board, 6 ops per byte",
+                         "kernel_ms_per_search": exp_ms,
+                         "peak_from": f"{SM_COUNT_GB300} SMs x {INT_LANES_PER_SM} int32 lanes/clk"
+                                      f" x {sm_max:.0f} MHz (sm_max_mhz of measured peaks)"},
+            "gpu_launches": args.steps * (1 + 2 * iters),
+            "wall_s_timed_region": wall,
+        }
+        if clocks:
+            line["clocks"] = clocks
+        if world == 1 and not args.no_cpu_baseline:
+            import oracle
+            cfg = oracle.make_cfg(**fields)
+            line["cpu_baseline"] = search_cpu_baseline(wl, rules, cum, cfg, seed)
+        print(json.dumps(line))
+    env.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def search_cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0) -> dict:
+    """The oracle's search, all host cores, on a bounded sample of envs."""
+    import oracle
+    threads = os.cpu_count() or 1
+    s = wk.seeds(seed)
+    n = min(wl.batch, max(threads, 4))
+    while True:
+        ids = np.arange(n)
+        roots = oracle.reset(cfg, cum, s["reset"], ids)
+        t0 = time.perf_counter()
+        ref = oracle.search(cfg, rules, roots, wl.iterations, wl.frontier, env_ids=ids,
+                            threads=threads)
+        dt = time.perf_counter() - t0
+        if dt > budget_s / 4 or n >= wl.batch:
+            break
+        n = min(wl.batch, int(n * max(2.0, budget_s / 4 / max(dt, 1e-3))))
+    children = 5 * (n + int(ref["trace_n"][:, :-1].sum()))
+    return {"value": children / dt, "unit": "env-steps/s", "cores": threads, "kind": "oracle",
+            "sample": f"{n} of {wl.batch} envs, full search ({wl.iterations} iterations,"
+                      f" frontier {wl.frontier})", "seconds": dt}
+
+
+def run_search_reference(args, wl):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    _, rules, cum = wk.make(wl, args.seed)
+    fields = wk.config_fields(wl)
+    cfg = oracle.make_cfg(**fields)
+    threads = os.cpu_count() or 1
+    s = wk.seeds(args.seed)
+    n = min(wl.batch, max(threads, 4))
+    ids = np.arange(n)
+    roots = oracle.reset(cfg, cum, s["reset"], ids)
+    for _ in range(args.warmup):
+        oracle.search(cfg, rules, roots, 2, wl.frontier, env_ids=ids, threads=threads)
+    times, children = [], 0
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        ref = oracle.search(cfg, rules, roots, wl.iterations, wl.frontier, env_ids=ids,
+                            threads=threads)
+        times.append(time.perf_counter() - t0)
+        children = 5 * (n + int(ref["trace_n"][:, :-1].sum()))
+    mean = sum(times) / len(times)
+    value = children / mean
+    line = {
+        "impl": "reference", "metric": "env-steps/s", "value": value, "unit": "env-steps/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+        "data": "synthetic", "config": dict(config_dict(wl, sample=n), frontier=wl.frontier,
+                                            iterations=wl.iterations),
+        "cpu_baseline": {"value": value, "unit": "env-steps/s", "cores": threads,
+                         "kind": "oracle",
+                         "sample": f"{n} of {wl.batch} envs, full search per step"},
+        "e2e": {"value": value, "unit": "env-steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
 def run_int_probe() -> int:
     """Build and run the integer-issue probe (needs nvcc and a GPU)."""
     import tempfile
@@ -433,7 +670,7 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--config", type=int, default=2, choices=(2, 3, 5))
+    ap.add_argument("--config", type=int, default=2, choices=(2, 3, 4, 5))
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--int-probe", action="store_true", help="measure integer issue rate and exit")
@@ -443,6 +680,8 @@ def main(argv=None):
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     wl = workload_for(args.config)
+    if wl.frontier:
+        return run_search_reference(args, wl) if args.impl == "reference" else run_search(args, wl)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_ours(args, wl)

@@ -127,6 +127,7 @@ class Workload:
     trajectory: bool = False  # rollout also writes obs/reward/done per step
     frontier: int = 0  # search: nodes kept per env (top-k)
     iterations: int = 0  # search: expand+select iterations
+    base_game: bool = False  # rules 0 and 1 of every table: the maze game's move and eat
 
     @property
     def nch(self) -> int:
@@ -149,7 +150,7 @@ WORKLOADS = {
                 ((1, 2), (1, 3), (3, 3)), 0.15, 0.15, 0.1, 0.1, -3, 3, steps=2000,
                 max_steps=200, auto_reset=1, trajectory=True),
     4: Workload(4, "search16-b64-f256-c8-r8", 64, 16, 16, 8, 8, ((3, 3),), 0.15, 0.15,
-                0.1, 0.1, -3, 3, frontier=256, iterations=50),
+                0.1, 0.1, -3, 3, init="maze", frontier=256, iterations=50, base_game=True),
     5: Workload(5, "grid64-b4096-c16-r24", 4096, 64, 64, 16, 24, ((3, 3), (5, 5)), 0.1,
                 0.1, 0.1, 0.1, -5, 5, steps=500),
 }
@@ -204,7 +205,28 @@ def make_rules(wl: Workload, seed: int, env_chunk: int = 2048) -> np.ndarray:
         blk["absent"] = absent
         blk["set"] = setm
         blk["clear"] = clrm
+    if wl.base_game and R >= 2:
+        out[:, 0:2] = base_game_rules(C)
     return out
+
+
+def base_game_rules(C: int) -> np.ndarray:
+    """The maze game every evolved environment starts from (Sec. 2.2.1): the
+    player moves onto floor where it pushes the force tile (Sec. 2.1, movement
+    paragraph), and moving onto a food tile eats it for a reward of 1."""
+    r = np.zeros(2, dtype=RULE_DTYPE)
+    P, E, G, F = 1 << CH_PLAYER, 1 << CH_EMPTY, 1 << CH_GOAL, 1 << C
+    for j in range(2):
+        r[j]["h"], r[j]["w"] = 1, 2
+        r[j]["present"][0] = P
+        r[j]["clear"][0] = P
+    r[0]["present"][1] = F | E  # move: player, then force on floor
+    r[0]["set"][1] = P
+    r[1]["present"][1] = F | G  # eat: player, then force on food
+    r[1]["set"][1] = P | E
+    r[1]["clear"][1] = G
+    r[1]["reward"] = 1
+    return r
 
 
 def make_init_cum(wl: Workload, seed: int) -> np.ndarray:
