@@ -160,7 +160,9 @@ int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_par
 /* Start a search from the root boards roots (device [B][H][W]): writes
  * root_hash uint64[B] (FNV-1a 64 as in av_expand) and root_live uint8[B]
  * (1 unless the root has no goal left), and sets the visited set of env b
- * to { root_hash[b] }.  AV_ESTATE if cfg.search_capacity < 1. */
+ * to { root_hash[b] }.  AV_ESTATE if cfg.search_capacity < 1.  The handle
+ * keeps each env's visited set as an open-addressing hash table of the
+ * smallest power of two >= max(64, 2 x search_capacity) 8-byte slots. */
 int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t *root_live,
                    uintptr_t stream);
 

@@ -39,9 +39,10 @@ struct av_handle {
     int32_t *d_t = nullptr;
     uint32_t *d_cum = nullptr;
     uint32_t *d_status = nullptr;  // [0] error bits, [1] warning bits
-    uint64_t *d_visited = nullptr;  // [2][B][capacity] sorted hashes (double-buffered)
+    uint64_t *d_vtab = nullptr;     // [B][vis_mask + 1] visited hashes, open addressing (0 = empty)
+    uint32_t *d_vzero = nullptr;    // [B] 1 if the state whose hash is 0 was visited
     int32_t *d_n_visited = nullptr; // [B]
-    int vis_parity = 0;
+    uint32_t vis_mask = 0;          // slots per env - 1 (a power of two >= 2 x capacity, minus one)
     bool has_cum = false;
     std::string last_error;
 };
@@ -359,7 +360,8 @@ void free_all(av_handle *h)
     cudaFree(h->d_t);
     cudaFree(h->d_cum);
     cudaFree(h->d_status);
-    cudaFree(h->d_visited);
+    cudaFree(h->d_vtab);
+    cudaFree(h->d_vzero);
     cudaFree(h->d_n_visited);
 }
 
@@ -509,7 +511,11 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
         h->has_cum = true;
     }
     if (cfg->search_capacity > 0) {
-        if ((rc = dalloc(h, &h->d_visited, 2 * B * (size_t)cfg->search_capacity)) ||
+        size_t slots = 64;
+        while (slots < 2 * (size_t)cfg->search_capacity)
+            slots <<= 1;
+        h->vis_mask = (uint32_t)(slots - 1);
+        if ((rc = dalloc(h, &h->d_vtab, B * slots)) || (rc = dalloc(h, &h->d_vzero, B)) ||
             (rc = dalloc(h, &h->d_n_visited, B))) {
             free_all(h);
             delete h;
@@ -634,9 +640,11 @@ int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t
         return AV_EINVAL;
     if (h->host_cfg.search_capacity < 1)
         return fail(h, AV_ESTATE, "av_search_init: search_capacity is 0");
-    h->vis_parity = 0;
-    launch_search_init(h->cf, h->host_cfg.search_capacity, roots, root_hash, root_live, h->d_visited,
-                       h->d_n_visited, as_stream(stream));
+    const cudaStream_t st = as_stream(stream);
+    AV_CUDA(h, cudaMemsetAsync(h->d_vtab, 0, (size_t)h->cf.B * (h->vis_mask + 1) * sizeof(uint64_t), st));
+    AV_CUDA(h, cudaMemsetAsync(h->d_vzero, 0, (size_t)h->cf.B * sizeof(uint32_t), st));
+    launch_search_init(h->cf, h->vis_mask, roots, root_hash, root_live, h->d_vtab, h->d_vzero, h->d_n_visited,
+                       st);
     return launch_check(h, "search init kernel");
 }
 
@@ -655,11 +663,10 @@ int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *p
     if (!n_parent || !parent_cum || !parent_live || !cand_grids || !cand_reward || !cand_done ||
         !cand_hash || !next_grids || !next_cum || !next_hash || !next_live || !n_next)
         return AV_EINVAL;
-    launch_select(h->cf, h->host_cfg.search_capacity, h->vis_parity, F, n_parent, parent_cum,
-                  parent_live, cand_grids, cand_reward, cand_done, cand_hash, k, next_grids,
-                  next_cum, next_hash, next_live, n_next, h->d_visited, h->d_n_visited,
-                  h->d_status, as_stream(stream));
-    h->vis_parity ^= 1;
+    launch_select_hash(h->cf, h->host_cfg.search_capacity, h->vis_mask, F, n_parent, parent_cum, parent_live,
+                       cand_grids, cand_reward, cand_done, cand_hash, k, next_grids, next_cum, next_hash,
+                       next_live, n_next, h->d_vtab, h->d_vzero, h->d_n_visited, h->d_status,
+                       as_stream(stream));
     return launch_check(h, "select kernel");
 }
 

@@ -1824,32 +1824,6 @@ reset_kernel(DevConfig cf, const uint32_t *__restrict__ cum_all, uint64_t seed, 
 }
 
 // --------------------------------------------------------------- search
-template <typename CellT>
-__global__ void search_init_kernel(DevConfig cf, int cap, const CellT *__restrict__ roots,
-                                   uint64_t *root_hash, uint8_t *root_live, uint64_t *visited,
-                                   int32_t *n_visited)
-{
-    const int b = blockIdx.x * blockDim.x + threadIdx.x;
-    if (b >= cf.B)
-        return;
-    const CellT *g = roots + (size_t)b * cf.HW;
-    const uint32_t tiles = (1u << cf.C) - 1u;
-    uint64_t hsh = 0xcbf29ce484222325ULL;
-    int goal = cf.ch_goal < 0;
-    for (int p = 0; p < cf.HW; ++p) {
-        const uint32_t v = (uint32_t)g[p] & tiles;
-        hsh = (hsh ^ (v & 0xffu)) * 0x100000001b3ULL;
-        if (sizeof(CellT) == 2)
-            hsh = (hsh ^ (v >> 8)) * 0x100000001b3ULL;
-        if (cf.ch_goal >= 0)
-            goal |= (int)((v >> cf.ch_goal) & 1u);
-    }
-    root_hash[b] = hsh;
-    root_live[b] = (uint8_t)goal;
-    visited[(size_t)b * cap] = hsh;  // parity 0
-    n_visited[b] = 1;
-}
-
 struct Key128 {
     uint64_t hi, lo;
 };
@@ -2025,6 +1999,230 @@ select_kernel(DevConfig cf, int cap, int parity, int F, const int32_t *__restric
         vis_out[i + lower_bound_u64(sel, take, vis_in[i])] = vis_in[i];
     for (int j = tid; j < take; j += blockDim.x)
         vis_out[j + lower_bound_u64(vis_in, nv, sel[j])] = sel[j];
+    if (tid == 0)
+        n_visited[b] = nv + take;
+}
+
+// ------------------------------------------------- selection with hash tables
+// av_select on a handle.  The visited states of env b live in an
+// open-addressing table vtab[b][0, T) of 64-bit hashes (T a power of two with
+// T >= 2 x capacity, so it is at most half full and every probe sequence ends
+// at an empty slot); 0 marks an empty slot and vzero[b] records the state
+// whose hash is 0.  A probe starts at mix64(hash) mod T and walks forward.
+// One CTA per env:
+//   1. each candidate that exists and is not visited goes into a shared-memory
+//      table keyed by hash, keeping per hash the smallest (cum desc, index),
+//      i.e. the highest cumulative reward and then the lowest index;
+//   2. the distinct candidates are compacted and sorted once by (cum desc,
+//      hash asc); the first k form the next frontier;
+//   3. their hashes are added to the visited table (all are new: step 1 kept
+//      only states not visited, one per hash).
+// The result is the selection the sorted-array kernel (select_kernel) makes.
+
+__device__ __forceinline__ uint32_t vis_slot(uint64_t h, uint32_t mask) { return (uint32_t)mix64(h) & mask; }
+
+__device__ __forceinline__ bool vis_contains(const uint64_t *tab, uint32_t mask, uint32_t zero, uint64_t h)
+{
+    if (h == 0)
+        return zero != 0u;
+    uint32_t slot = vis_slot(h, mask);
+    for (uint32_t probe = 0; probe <= mask; ++probe) {
+        const uint64_t v = tab[slot];
+        if (v == h)
+            return true;
+        if (v == 0)
+            return false;
+        slot = (slot + 1) & mask;
+    }
+    return false;
+}
+
+// Insert h (not present, nonzero) into a table with a free slot.
+__device__ __forceinline__ void vis_insert(uint64_t *tab, uint32_t mask, uint64_t h)
+{
+    uint32_t slot = vis_slot(h, mask);
+    for (uint32_t probe = 0; probe <= mask; ++probe) {
+        const unsigned long long prev =
+            atomicCAS(reinterpret_cast<unsigned long long *>(tab + slot), 0ull, (unsigned long long)h);
+        if (prev == 0ull || prev == (unsigned long long)h)
+            return;
+        slot = (slot + 1) & mask;
+    }
+}
+
+template <typename CellT>
+__global__ void __launch_bounds__(kThreads)
+search_init_hash_kernel(DevConfig cf, uint32_t vmask, const CellT *__restrict__ roots, uint64_t *root_hash,
+                        uint8_t *root_live, uint64_t *vtab, uint32_t *vzero, int32_t *n_visited)
+{
+    // one thread per env; the tables were cleared before the launch
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= cf.B)
+        return;
+    const CellT *g = roots + (size_t)b * cf.HW;
+    const uint32_t tiles = (1u << cf.C) - 1u;
+    uint64_t hsh = 0xcbf29ce484222325ULL;
+    int goal = cf.ch_goal < 0;
+    for (int p = 0; p < cf.HW; ++p) {
+        const uint32_t v = (uint32_t)g[p] & tiles;
+        hsh = (hsh ^ (v & 0xffu)) * 0x100000001b3ULL;
+        if (sizeof(CellT) == 2)
+            hsh = (hsh ^ (v >> 8)) * 0x100000001b3ULL;
+        if (cf.ch_goal >= 0)
+            goal |= (int)((v >> cf.ch_goal) & 1u);
+    }
+    root_hash[b] = hsh;
+    root_live[b] = (uint8_t)goal;
+    if (hsh == 0)
+        vzero[b] = 1u;
+    else
+        vis_insert(vtab + (size_t)b * (vmask + 1), vmask, hsh);
+    n_visited[b] = 1;
+}
+
+// Shared memory of select_hash_kernel for 5 * F candidates.
+__host__ __device__ inline uint32_t select_hash_slots(int F)
+{
+    uint32_t t = 64;
+    while (t < 2u * 5u * (uint32_t)F)
+        t <<= 1;
+    return t;
+}
+inline size_t select_hash_smem_bytes(int F)
+{
+    int n2 = 1;
+    while (n2 < 5 * F)
+        n2 <<= 1;
+    return (size_t)select_hash_slots(F) * 16 + (size_t)n2 * sizeof(Key128) + 64;
+}
+
+template <typename CellT>
+__global__ void __launch_bounds__(kThreads)
+select_hash_kernel(DevConfig cf, int cap, uint32_t vmask, int F, const int32_t *__restrict__ n_parent,
+                   const int32_t *__restrict__ parent_cum, const uint8_t *__restrict__ parent_live,
+                   const CellT *__restrict__ cand_grids, const int32_t *__restrict__ cand_reward,
+                   const uint8_t *__restrict__ cand_done, const uint64_t *__restrict__ cand_hash, int k,
+                   CellT *next_grids, int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live,
+                   int32_t *n_next, uint64_t *vtab, uint32_t *vzero, int32_t *n_visited, uint32_t *status)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    const uint32_t T = select_hash_slots(F), smask = T - 1;
+    unsigned long long *skey = reinterpret_cast<unsigned long long *>(smem);
+    unsigned long long *sval = skey + T;
+    Key128 *keys = reinterpret_cast<Key128 *>(sval + T);
+    __shared__ unsigned long long s_zero_val;
+    __shared__ int s_count;
+    const int b = blockIdx.x, tid = threadIdx.x, HW = cf.HW;
+    const int nc = 5 * F;
+    const uint64_t *vt = vtab + (size_t)b * (vmask + 1);
+    const uint32_t vz = vzero[b];
+    const int np = n_parent[b];
+
+    for (uint32_t i = tid; i < T; i += blockDim.x) {
+        skey[i] = 0ull;
+        sval[i] = ~0ull;
+    }
+    if (tid == 0) {
+        s_zero_val = ~0ull;
+        s_count = 0;
+    }
+    __syncthreads();
+
+    // 1. candidates that exist and are not yet visited, one per hash
+    for (int i = tid; i < nc; i += blockDim.x) {
+        const int f = i / 5;
+        const size_t gi = (size_t)b * F + f;
+        if (f >= np || !parent_live[gi])
+            continue;
+        const uint64_t hsh = cand_hash[(size_t)b * nc + i];
+        if (vis_contains(vt, vmask, vz, hsh))
+            continue;
+        const int32_t cum = parent_cum[gi] + cand_reward[(size_t)b * nc + i];
+        const unsigned long long packed = ((unsigned long long)cum_desc_key(cum) << 32) | (uint32_t)i;
+        if (hsh == 0) {
+            atomicMin(&s_zero_val, packed);
+            continue;
+        }
+        uint32_t slot = vis_slot(hsh, smask);
+        for (uint32_t probe = 0; probe <= smask; ++probe) {
+            const unsigned long long prev = atomicCAS(&skey[slot], 0ull, (unsigned long long)hsh);
+            if (prev == 0ull || prev == (unsigned long long)hsh) {
+                atomicMin(&sval[slot], packed);
+                break;
+            }
+            slot = (slot + 1) & smask;
+        }
+    }
+    __syncthreads();
+
+    // 2. distinct candidates keyed (cum desc, hash, index); one sort
+    for (uint32_t i = tid; i <= T; i += blockDim.x) {
+        uint64_t hsh;
+        unsigned long long v;
+        if (i < T) {
+            hsh = skey[i];
+            v = sval[i];
+            if (hsh == 0ull)
+                continue;
+        } else {
+            v = s_zero_val;
+            hsh = 0ull;
+            if (v == ~0ull)
+                continue;
+        }
+        const int pos = atomicAdd(&s_count, 1);
+        keys[pos].hi = ((v >> 32) << 32) | (hsh >> 32);
+        keys[pos].lo = (hsh << 32) | (v & 0xffffffffull);
+    }
+    __syncthreads();
+    const int nu = s_count;
+    int n2 = 1;
+    while (n2 < nu)
+        n2 <<= 1;
+    for (int i = nu + tid; i < n2; i += blockDim.x)
+        keys[i] = Key128{~0ull, ~0ull};
+    __syncthreads();
+    bitonic_sort(keys, n2);
+    const int take = min(k, nu);
+
+    // 3. next frontier
+    for (int s = tid; s < take; s += blockDim.x) {
+        const Key128 x = keys[s];
+        const int idx = (int)(x.lo & 0xffffffffull);
+        const uint64_t hsh = (x.hi << 32) | (x.lo >> 32);
+        const size_t gi = (size_t)b * F + idx / 5;
+        next_cum[(size_t)b * k + s] = parent_cum[gi] + cand_reward[(size_t)b * nc + idx];
+        next_hash[(size_t)b * k + s] = hsh;
+        next_live[(size_t)b * k + s] = (uint8_t)!cand_done[(size_t)b * nc + idx];
+    }
+    for (int s = take + tid; s < k; s += blockDim.x) {
+        next_cum[(size_t)b * k + s] = 0;
+        next_hash[(size_t)b * k + s] = 0;
+        next_live[(size_t)b * k + s] = 0;
+    }
+    for (int e = tid; e < take * HW; e += blockDim.x) {
+        const int s = e / HW, p = e - s * HW;
+        const int idx = (int)(keys[s].lo & 0xffffffffull);
+        next_grids[((size_t)b * k + s) * HW + p] = cand_grids[((size_t)b * nc + idx) * HW + p];
+    }
+    if (tid == 0)
+        n_next[b] = take;
+
+    // 4. the selected states join the visited set
+    const int nv = n_visited[b];
+    if (nv + take > cap) {
+        if (tid == 0)
+            atomicOr(status, kStatusVisitedOverflow);
+        return;  // the set stays as it was, as with the sorted arrays
+    }
+    uint64_t *vw = vtab + (size_t)b * (vmask + 1);
+    for (int s = tid; s < take; s += blockDim.x) {
+        const uint64_t hsh = (keys[s].hi << 32) | (keys[s].lo >> 32);
+        if (hsh == 0)
+            vzero[b] = 1u;
+        else
+            vis_insert(vw, vmask, hsh);
+    }
     if (tid == 0)
         n_visited[b] = nv + take;
 }

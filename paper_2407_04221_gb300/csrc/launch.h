@@ -49,8 +49,15 @@ void launch_expand(const DevConfig &cf, const uint32_t *arena, const uint32_t *t
                    int32_t *rewards, uint8_t *done, uint64_t *hashes, cudaStream_t st);
 void launch_reset(const DevConfig &cf, const uint32_t *cum, uint64_t seed, void *cur, void *init, int32_t *t,
                   void *obs, cudaStream_t st);
-void launch_search_init(const DevConfig &cf, int cap, const void *roots, uint64_t *root_hash,
-                        uint8_t *root_live, uint64_t *visited, int32_t *n_visited, cudaStream_t st);
+void launch_search_init(const DevConfig &cf, uint32_t vmask, const void *roots, uint64_t *root_hash,
+                        uint8_t *root_live, uint64_t *vtab, uint32_t *vzero, int32_t *n_visited,
+                        cudaStream_t st);
+void launch_select_hash(const DevConfig &cf, int cap, uint32_t vmask, int F, const int32_t *n_parent,
+                        const int32_t *parent_cum, const uint8_t *parent_live, const void *cand_grids,
+                        const int32_t *cand_reward, const uint8_t *cand_done, const uint64_t *cand_hash, int k,
+                        void *next_grids, int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live,
+                        int32_t *n_next, uint64_t *vtab, uint32_t *vzero, int32_t *n_visited, uint32_t *status,
+                        cudaStream_t st);
 void launch_select(const DevConfig &cf, int cap, int parity, int F, const int32_t *n_parent,
                    const int32_t *parent_cum, const uint8_t *parent_live, const void *cand_grids,
                    const int32_t *cand_reward, const uint8_t *cand_done, const uint64_t *cand_hash, int k,
