@@ -8,8 +8,15 @@ namespace {
 #define AV_FOR_NA(MACRO, CELL) MACRO(CELL, 1) MACRO(CELL, 2) MACRO(CELL, 4) MACRO(CELL, 8) MACRO(CELL, 16)
 
 // Parents per CTA on the warp path: 1 while the GPU has room for every warp at
-// once (best balance), more for large batches.
-int warps_per_cta(long long units) { return units <= 152LL * 32 ? 1 : (units <= 152LL * 64 ? 2 : kWarpCtaMax); }
+// once (best balance), more for large batches.  The count divides F so that
+// a CTA's parents share one environment (and its rule table).
+int warps_per_cta(long long units, int F)
+{
+    int w = units <= 152LL * 32 ? 1 : (units <= 152LL * 64 ? 2 : kWarpCtaMax);
+    while (w > 1 && F % w != 0)
+        w >>= 1;
+    return w;
+}
 
 template <typename CellT, int NA>
 void block_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
@@ -34,9 +41,10 @@ void warp_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
             int32_t *rewards, uint8_t *done, uint64_t *hashes, cudaStream_t st)
 {
     const long long units = (long long)cf.B * F;
-    const int wpc = warps_per_cta(units);
+    const int wpc = warps_per_cta(units, F);
     const unsigned grid = (unsigned)((units + wpc - 1) / wpc);
-    const size_t sm = (size_t)wpc * warp_layout(cf, 5).total;
+    const ExpandLayout L = expand_layout(cf);
+    const size_t sm = L.warps + (size_t)wpc * L.per_warp;
     if (cf.rule_words > 0)
         expand_warp_kernel<CellT, NA, RB, true><<<grid, 32 * wpc, sm, st>>>(
             cf, arena, tab_off, vm, masks, (const CellT *)parents, F, n_parent, (CellT *)children, rewards,

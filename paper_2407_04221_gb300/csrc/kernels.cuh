@@ -582,7 +582,7 @@ expand_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *
 // (independent dependency chains), continues only the rules that still have a
 // live anchor, and then updates its board itself: no block-wide barrier.
 
-constexpr int kWarpCtaMax = 4;  // warps (= environments) per CTA at most
+constexpr int kWarpCtaMax = 8;  // warps (= parents) per CTA at most
 
 struct WarpLayout {
     size_t planes, setp, clrp, basep, vm, masks, acts, rules, cells, total;
@@ -821,6 +821,71 @@ __device__ __forceinline__ void warp_combine(const DevConfig &cf, const WarpSmem
     }
 }
 
+// Shared memory of expand_warp_kernel: one region per CTA (the rule table when
+// staged, valid-anchor masks, column masks), then per warp its planes, SET /
+// CLEAR / child planes and the canonical bytes of its five children.  All
+// warps of a CTA expand parents of one environment (the host makes the warp
+// count divide F), so they share the table.
+struct ExpandLayout {
+    size_t vm, masks, rules, warps;  // CTA region
+    size_t planes, setp, clrp, basep, bytes, per_warp;  // offsets within a warp's region
+    size_t child_bytes;  // canonical bytes of one child, padded to 16
+};
+
+__host__ __device__ inline ExpandLayout expand_layout(const DevConfig &cf)
+{
+    ExpandLayout L;
+    const size_t pw = (size_t)cf.C * cf.NW * 4;
+    L.vm = 0;
+    L.masks = align16((size_t)kShapes * cf.NW * 4);
+    L.rules = align16(L.masks + (size_t)3 * cf.NW * 4);
+    L.warps = align16(L.rules + (size_t)cf.rule_words * 4);
+    L.child_bytes = align16((size_t)cf.HW * cf.cell_bytes);
+    L.planes = 0;
+    L.setp = align16((size_t)(cf.C + 1) * cf.NWP * 8);
+    L.clrp = align16(L.setp + pw);
+    L.basep = align16(L.clrp + pw);
+    L.bytes = align16(L.basep + pw);
+    L.per_warp = align16(L.bytes + 5 * L.child_bytes);
+    return L;
+}
+
+// Cells of a board from its flat planes (C words per plane word), written as
+// canonical bytes to `out` (shared, 16-byte aligned) and to `dst` (global),
+// and whether any goal tile is left.  One warp; a 32-bit word per lane per
+// pass: four 1-byte cells (bit k of a channel's 4-bit slice spread to byte k
+// by a multiply) or two 2-byte cells.
+template <typename CellT>
+__device__ __forceinline__ int planes_to_cells(const DevConfig &cf, const uint32_t *flat, uint32_t *out,
+                                               CellT *dst)
+{
+    const int lane = threadIdx.x & 31, HW = cf.HW, NW = cf.NW;
+    constexpr int kPer = 4 / (int)sizeof(CellT);  // cells per 32-bit word
+    const int n_words = (HW + kPer - 1) / kPer;
+    const bool aligned = (HW % kPer) == 0 && (reinterpret_cast<uintptr_t>(dst) & 3u) == 0;
+    int goal = 0;
+    for (int g = lane; g < n_words; g += 32) {
+        const int p0 = g * kPer, j = p0 >> 5, b = p0 & 31;
+        uint32_t v = 0;
+        for (int c = 0; c < cf.C; ++c) {
+            const uint32_t x = flat[c * NW + j] >> b;
+            const uint32_t spread = sizeof(CellT) == 1 ? ((x & 0xfu) * 0x00204081u) & 0x01010101u
+                                                       : ((x & 0x3u) * 0x00008001u) & 0x00010001u;
+            v |= spread << c;
+        }
+        out[g] = v;
+        if (cf.ch_goal >= 0)
+            goal |= (int)(((v >> cf.ch_goal) & (sizeof(CellT) == 1 ? 0x01010101u : 0x00010001u)) != 0u);
+        if (aligned) {
+            reinterpret_cast<uint32_t *>(dst)[g] = v;
+        } else {
+            for (int k = 0; k < kPer && p0 + k < HW; ++k)
+                dst[p0 + k] = (CellT)(v >> (8 * (int)sizeof(CellT) * k));
+        }
+    }
+    return __any_sync(0xffffffffu, goal) || cf.ch_goal < 0;
+}
+
 template <typename CellT, int NA, int RB, bool SM>
 __global__ void __launch_bounds__(32 * kWarpCtaMax)
 expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
@@ -829,69 +894,118 @@ expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint3
                    CellT *children, int32_t *rewards, uint8_t *done, uint64_t *hashes)
 {
     extern __shared__ __align__(16) unsigned char smem[];
-    const long long node = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (node >= (long long)cf.B * F)
-        return;
-    const int env = (int)(node / F);
-    if (n_parent && (int)(node - (long long)env * F) >= n_parent[env])
-        return;  // an empty frontier slot
-    const int lane = threadIdx.x & 31, HW = cf.HW, NW = cf.NW, NWP = cf.NWP, C = cf.C;
-    const WarpSmem S = carve_warp(smem, cf, 5);
-    const int table = cf.rules_per_env ? env : 0;
-    const uint32_t *tab_g = arena + tab_off[table];
-    const uint32_t *tab = SM ? S.rules : tab_g;
+    const ExpandLayout L = expand_layout(cf);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+    const long long first = (long long)blockIdx.x * nwarps;  // this CTA's first parent
+    const long long node = first + warp;
+    const long long total = (long long)cf.B * F;
+    const int env0 = (int)(min(first, total - 1) / F);
+    bool mine = node < total;  // this warp has a parent to expand
+    const int env = mine ? (int)(node / F) : env0;
+    if (mine && n_parent && (int)(node - (long long)env * F) >= n_parent[env])
+        mine = false;  // an empty frontier slot
+    const int HW = cf.HW, NW = cf.NW, NWP = cf.NWP, C = cf.C;
 
-    warp_stage(cf, S, vm_g, masks_g, tab_g, tab_off[table + 1] - tab_off[table], SM);
-    warp_cells_to_planes<CellT>(cf, parents + (size_t)node * HW, S.planes, nullptr);
-    __syncwarp();
-    for (int a = 0; a < 5; ++a) {
-        force_plane(cf, S.planes, S.masks, a);
-        __syncwarp();
-        const int2 o = warp_rules<NA, RB, SM>(cf, tab, S);
-        const int rew = __reduce_add_sync(0xffffffffu, o.x);
-        __syncwarp();
-        const bool any = __any_sync(0xffffffffu, o.y != 0);
-        for (int i = lane; i < C * NW; i += 32) {  // child planes
-            const int c = i / NW, w = i - c * NW;
-            const uint32_t d = S.planes[c * NWP + w].x;
-            uint32_t v = d;
-            if (any) {
-                v = (d & ~S.clrp[i]) | (~d & S.setp[i]);
-                S.setp[i] = 0u;
-                S.clrp[i] = 0u;
-            }
-            S.basep[i] = v;
-        }
-        __syncwarp();
-        uint16_t *cells = S.cells + (size_t)a * HW;
-        CellT *dst = children + ((size_t)node * 5 + a) * HW;
-        int goal = 0;
-        for (int p = lane; p < HW; p += 32) {
-            const uint32_t v = gather_cell(cf, nullptr, S.basep, p);
-            cells[p] = (uint16_t)v;
-            dst[p] = (CellT)v;
-            if (cf.ch_goal >= 0)
-                goal |= (int)((v >> cf.ch_goal) & 1u);
-        }
-        const int goal_left = __any_sync(0xffffffffu, goal) || cf.ch_goal < 0;
-        if (lane == 0) {
-            rewards[(size_t)node * 5 + a] = rew;
-            if (done)
-                done[(size_t)node * 5 + a] = (uint8_t)!goal_left;
-        }
-        __syncwarp();
+    // ---- the CTA's shared region
+    uint32_t *vm = reinterpret_cast<uint32_t *>(smem + L.vm);
+    uint32_t *masks = reinterpret_cast<uint32_t *>(smem + L.masks);
+    uint32_t *rules = reinterpret_cast<uint32_t *>(smem + L.rules);
+    const int table = cf.rules_per_env ? env0 : 0;
+    const uint32_t *tab_g = arena + tab_off[table];
+    for (int i = threadIdx.x; i < kShapes * NW; i += blockDim.x)
+        vm[i] = __ldg(vm_g + i);
+    for (int i = threadIdx.x; i < 3 * NW; i += blockDim.x)
+        masks[i] = __ldg(masks_g + i);
+    if (SM) {
+        const uint32_t n = tab_off[table + 1] - tab_off[table];
+        const uint4 *src = reinterpret_cast<const uint4 *>(tab_g);
+        uint4 *d = reinterpret_cast<uint4 *>(rules);
+        for (uint32_t i = threadIdx.x; i < n / 4; i += blockDim.x)
+            d[i] = __ldg(src + i);
     }
-    // FNV-1a 64 over the canonical bytes, one lane per child
-    if (lane < 5) {
-        const uint16_t *gc = S.cells + (size_t)lane * HW;
-        uint64_t hsh = 0xcbf29ce484222325ULL;
-        for (int p = 0; p < HW; ++p) {
-            const uint32_t v = gc[p];
-            hsh = (hsh ^ (v & 0xffu)) * 0x100000001b3ULL;
-            if (sizeof(CellT) == 2)
-                hsh = (hsh ^ (v >> 8)) * 0x100000001b3ULL;
+    // ---- this warp's region
+    unsigned char *wr = smem + L.warps + (size_t)warp * L.per_warp;
+    WarpSmem S;
+    S.planes = reinterpret_cast<uint2 *>(wr + L.planes);
+    S.setp = reinterpret_cast<uint32_t *>(wr + L.setp);
+    S.clrp = reinterpret_cast<uint32_t *>(wr + L.clrp);
+    S.basep = reinterpret_cast<uint32_t *>(wr + L.basep);
+    S.vm = vm;
+    S.masks = masks;
+    S.rules = rules;
+    S.acts = nullptr;
+    S.cells = nullptr;
+    uint32_t *bytes = reinterpret_cast<uint32_t *>(wr + L.bytes);
+    const uint32_t *tab = SM ? rules : tab_g;
+    for (int i = lane; i < (C + 1) * NWP; i += 32)
+        S.planes[i] = make_uint2(0u, 0u);
+    for (int i = lane; i < C * NW; i += 32) {
+        S.setp[i] = 0u;
+        S.clrp[i] = 0u;
+    }
+    __syncthreads();  // the shared region
+
+    if (mine) {
+        warp_cells_to_planes<CellT>(cf, parents + (size_t)node * HW, S.planes, nullptr);
+        __syncwarp();
+        for (int a = 0; a < 5; ++a) {
+            force_plane(cf, S.planes, S.masks, a);
+            __syncwarp();
+            const int2 o = warp_rules<NA, RB, SM>(cf, tab, S);
+            const int rew = __reduce_add_sync(0xffffffffu, o.x);
+            __syncwarp();
+            const bool any = __any_sync(0xffffffffu, o.y != 0);
+            for (int i = lane; i < C * NW; i += 32) {  // child planes
+                const int c = i / NW, w = i - c * NW;
+                const uint32_t d = S.planes[c * NWP + w].x;
+                uint32_t v = d;
+                if (any) {
+                    v = (d & ~S.clrp[i]) | (~d & S.setp[i]);
+                    S.setp[i] = 0u;
+                    S.clrp[i] = 0u;
+                }
+                S.basep[i] = v;
+            }
+            __syncwarp();
+            const int goal_left = planes_to_cells<CellT>(
+                cf, S.basep, bytes + a * (L.child_bytes / 4), children + ((size_t)node * 5 + a) * HW);
+            if (lane == 0) {
+                rewards[(size_t)node * 5 + a] = rew;
+                if (done)
+                    done[(size_t)node * 5 + a] = (uint8_t)!goal_left;
+            }
+            __syncwarp();
         }
-        hashes[(size_t)node * 5 + lane] = hsh;
+    }
+    __syncthreads();  // every child's bytes
+
+    // ---- FNV-1a 64 over each child's canonical bytes, one thread per child
+    const int nbytes = HW * (int)sizeof(CellT);
+    for (int t = threadIdx.x; t < 5 * nwarps; t += blockDim.x) {
+        const int w = t / 5, a = t - 5 * w;
+        const long long nd = first + w;
+        if (nd >= total)
+            continue;
+        const int e = (int)(nd / F);
+        if (n_parent && (int)(nd - (long long)e * F) >= n_parent[e])
+            continue;
+        const uint32_t *cb = reinterpret_cast<const uint32_t *>(smem + L.warps + (size_t)w * L.per_warp + L.bytes) +
+                             a * (L.child_bytes / 4);
+        uint64_t hsh = 0xcbf29ce484222325ULL;
+        int k = 0;
+        for (; k + 4 <= nbytes; k += 4) {
+            const uint32_t x = cb[k >> 2];
+            hsh = (hsh ^ (x & 0xffu)) * 0x100000001b3ULL;
+            hsh = (hsh ^ ((x >> 8) & 0xffu)) * 0x100000001b3ULL;
+            hsh = (hsh ^ ((x >> 16) & 0xffu)) * 0x100000001b3ULL;
+            hsh = (hsh ^ (x >> 24)) * 0x100000001b3ULL;
+        }
+        if (k < nbytes) {
+            const uint32_t x = cb[k >> 2];
+            for (int r = 0; k + r < nbytes; ++r)
+                hsh = (hsh ^ ((x >> (8 * r)) & 0xffu)) * 0x100000001b3ULL;
+        }
+        hashes[(size_t)nd * 5 + a] = hsh;
     }
 }
 
