@@ -2314,10 +2314,23 @@ select_hash_kernel(DevConfig cf, int cap, uint32_t vmask, int F, const int32_t *
         next_hash[(size_t)b * k + s] = 0;
         next_live[(size_t)b * k + s] = 0;
     }
-    for (int e = tid; e < take * HW; e += blockDim.x) {
-        const int s = e / HW, p = e - s * HW;
-        const int idx = (int)(keys[s].lo & 0xffffffffull);
-        next_grids[((size_t)b * k + s) * HW + p] = cand_grids[((size_t)b * nc + idx) * HW + p];
+    const size_t board = (size_t)HW * sizeof(CellT);
+    if (board % 16 == 0 && (reinterpret_cast<uintptr_t>(cand_grids) & 15u) == 0 &&
+        (reinterpret_cast<uintptr_t>(next_grids) & 15u) == 0) {
+        const int n16 = (int)(board / 16);  // 16-byte pieces per board
+        const uint4 *src = reinterpret_cast<const uint4 *>(cand_grids);
+        uint4 *dst = reinterpret_cast<uint4 *>(next_grids);
+        for (int e = tid; e < take * n16; e += blockDim.x) {
+            const int s = e / n16, p = e - s * n16;
+            const int idx = (int)(keys[s].lo & 0xffffffffull);
+            dst[((size_t)b * k + s) * n16 + p] = src[((size_t)b * nc + idx) * n16 + p];
+        }
+    } else {
+        for (int e = tid; e < take * HW; e += blockDim.x) {
+            const int s = e / HW, p = e - s * HW;
+            const int idx = (int)(keys[s].lo & 0xffffffffull);
+            next_grids[((size_t)b * k + s) * HW + p] = cand_grids[((size_t)b * nc + idx) * HW + p];
+        }
     }
     if (tid == 0)
         n_next[b] = take;
