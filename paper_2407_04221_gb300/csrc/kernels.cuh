@@ -241,6 +241,37 @@ __device__ __forceinline__ uint32_t gather_cell(const DevConfig &cf, const uint2
     return v;
 }
 
+// Cells of a board from its doubled planes, stored to dst (global) a 32-bit
+// word at a time by threads tid, tid + nthreads, ...: four 1-byte cells (bit k
+// of a channel's 4-bit slice spread to byte k by a multiply) or two 2-byte
+// cells.  Falls back to one cell per store when dst is not 4-byte aligned or
+// the board does not fill whole words.
+template <typename CellT>
+__device__ __forceinline__ void store_cells(const DevConfig &cf, const uint2 *dbl, CellT *dst, int tid,
+                                            int nthreads)
+{
+    constexpr int kPer = 4 / (int)sizeof(CellT);
+    const int HW = cf.HW, NWP = cf.NWP;
+    const int n_words = (HW + kPer - 1) / kPer;
+    const bool aligned = (HW % kPer) == 0 && (reinterpret_cast<uintptr_t>(dst) & 3u) == 0;
+    for (int g = tid; g < n_words; g += nthreads) {
+        const int p0 = g * kPer, j = p0 >> 5, b = p0 & 31;
+        uint32_t v = 0;
+        for (int c = 0; c < cf.C; ++c) {
+            const uint32_t x = dbl[c * NWP + j].x >> b;
+            const uint32_t spread = sizeof(CellT) == 1 ? ((x & 0xfu) * 0x00204081u) & 0x01010101u
+                                                       : ((x & 0x3u) * 0x00008001u) & 0x00010001u;
+            v |= spread << c;
+        }
+        if (aligned) {
+            reinterpret_cast<uint32_t *>(dst)[g] = v;
+        } else {
+            for (int k = 0; k < kPer && p0 + k < HW; ++k)
+                dst[p0 + k] = (CellT)(v >> (8 * (int)sizeof(CellT) * k));
+        }
+    }
+}
+
 // Force plane for `action`, from the player plane (warp-cooperative, one warp).
 // Player at p puts force at p + d: d = -W up, +1 right, +W down, -1 left,
 // dropped where it would leave the board.
@@ -478,14 +509,10 @@ rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t 
         }
         __syncthreads();
         if (obs_traj) {
-            CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
-            for (int p = tid; p < HW; p += kThreads)
-                dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+            store_cells<CellT>(cf, S.planes, obs_traj + ((size_t)s * cf.B + env) * HW, tid, kThreads);
         }
     }
-    CellT *dst = cur + (size_t)env * HW;
-    for (int p = tid; p < HW; p += kThreads)
-        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+    store_cells<CellT>(cf, S.planes, cur + (size_t)env * HW, tid, kThreads);
     if (tid == 0) {
         tsteps[env] = t;
         if (rew_sum)
@@ -1412,15 +1439,11 @@ rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
             __syncthreads();
         }
         if (obs_traj) {
-            CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
-            for (int p = tid; p < HW; p += 32 * NWARP)
-                dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+            store_cells<CellT>(cf, S.planes, obs_traj + ((size_t)s * cf.B + env) * HW, tid, 32 * NWARP);
         }
         fdelta = fdelta_next;
     }
-    CellT *dst = cur + (size_t)env * HW;
-    for (int p = tid; p < HW; p += 32 * NWARP)
-        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+    store_cells<CellT>(cf, S.planes, cur + (size_t)env * HW, tid, 32 * NWARP);
     if (tid == 0) {
         tsteps[env] = t;
         if (rew_sum)
@@ -1538,6 +1561,79 @@ __device__ __forceinline__ int2 env_rule_rest(const DevConfig &cf, const uint32_
         }
     }
     return make_int2((int)h0.w * (int)cnt, 1);
+}
+
+// A general step's per-step outputs (one warp): reward and done flag, and the
+// board.  Not inlined: on one warp a branch around a large inline block costs
+// tens of cycles even when not taken, around a call a few.
+template <typename CellT>
+__device__ __noinline__ void env_step_outputs(DevConfig cf, const uint2 *planes, int env, int s, int rew,
+                                              int done, CellT *obs_traj, int32_t *rew_traj, uint8_t *done_traj)
+{
+    if ((threadIdx.x & 31) == 0) {
+        if (rew_traj)
+            rew_traj[(size_t)s * cf.B + env] = rew;
+        if (done_traj)
+            done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
+    }
+    if (obs_traj)
+        store_cells<CellT>(cf, planes, obs_traj + ((size_t)s * cf.B + env) * cf.HW, threadIdx.x & 31, 32);
+}
+
+// The board update of a general step in which a rule matched or a reset is
+// due (one warp): combine (a bit changes where any match asks for it), goal
+// test of the new board, auto-reset, the five force planes.  Returns (t,
+// goal_left, done).  Not inlined, like env_step_outputs.
+static __device__ __noinline__ int3 env_board_update(DevConfig cf, uint2 *planes, uint32_t *setp, uint32_t *clrp,
+                                                     const uint32_t *basep, const uint32_t *masks, int t)
+{
+    const int lane = threadIdx.x & 31, C = cf.C, NW = cf.NW, NWP = cf.NWP;
+    __syncwarp();  // every lane's SET / CLEAR bits
+    int gl = cf.ch_goal < 0;
+    for (int i = lane; i < C * NW; i += 32) {
+        const int c = i / NW, w = i - c * NW;
+        uint32_t d = planes[c * NWP + w].x;
+        const uint32_t st = setp[i], cl = clrp[i];
+        if (st | cl) {
+            setp[i] = 0u;
+            clrp[i] = 0u;
+            d = (d & ~cl) | (~d & st);
+            put_word(planes, NWP, c, w, d);
+        }
+        if (c == cf.ch_goal)
+            gl |= d != 0u;
+    }
+    int goal_left = __any_sync(0xffffffffu, gl);
+    int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+    if (done && cf.auto_reset) {
+        for (int i = lane; i < C * NW; i += 32) {
+            const int c = i / NW, w = i - c * NW;
+            put_word(planes, NWP, c, w, basep[i]);
+        }
+        t = 0;
+        gl = cf.ch_goal < 0;
+        if (cf.ch_goal >= 0)
+            for (int w = lane; w < NW; w += 32)
+                gl |= basep[cf.ch_goal * NW + w] != 0u;
+        goal_left = __any_sync(0xffffffffu, gl);
+    }
+    __syncwarp();  // the new board
+    force_planes(cf, planes, masks, 0, 1, C + 1);
+    __syncwarp();  // its force planes
+    return make_int3(t, goal_left, done);
+}
+
+// Actions [s + 128, s + 256) into the ring slots of steps [s - 128, s), all
+// read by now (one warp).  Not inlined, like env_step_outputs.
+static __device__ __noinline__ void env_refill(const uint8_t *actions, uint64_t seed, int env, int s, int n_steps,
+                                               uint8_t *acts, int *warn)
+{
+    const int lane = threadIdx.x & 31;
+    for (int k = lane; k < kActChunk / 2; k += 32)
+        if (s + kActChunk / 2 + k < n_steps)
+            acts[(s + kActChunk / 2 + k) & (kActChunk - 1)] =
+                (uint8_t)action_at(actions, seed, env, s + kActChunk / 2 + k, warn);
+    __syncwarp();
 }
 
 template <typename CellT, int NA, int RPW, bool SM>
@@ -1699,11 +1795,8 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
                     if (done_traj)
                         done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
                 }
-                if (obs_traj) {
-                    CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
-                    for (int p = lane; p < HW; p += 32)
-                        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
-                }
+                if (obs_traj)
+                    store_cells<CellT>(cf, S.planes, obs_traj + ((size_t)s * cf.B + env) * HW, lane, 32);
             }
             if (lane < NW)
                 slot[lane] = f_next;  // every read of this step's force is behind the vote
@@ -1718,11 +1811,7 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
         // actions [s + 128, s + 256) into the ring slots of steps [s - 128, s),
         // all read by now
         if (s > 0 && (s & (kActChunk / 2 - 1)) == 0 && s != refilled) {
-            for (int k = lane; k < kActChunk / 2; k += 32)
-                if (s + kActChunk / 2 + k < n_steps)
-                    S.acts[(s + kActChunk / 2 + k) & (kActChunk - 1)] =
-                        (uint8_t)action_at(actions, seed, env, s + kActChunk / 2 + k, S.ctl + 3);
-            __syncwarp();
+            env_refill(actions, seed, env, s, n_steps, S.acts, S.ctl + 3);
             refilled = s;
         }
         const int lim = min(n_steps, ((s / (kActChunk / 2)) + 1) * (kActChunk / 2));
@@ -1778,40 +1867,10 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
         t += 1;
         int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
         if (changed || (done && cf.auto_reset)) {
-            __syncwarp();  // every lane's SET / CLEAR bits
-            // combine: a bit changes where any match asks for it; the goal test
-            // of the new board comes with it
-            int gl = cf.ch_goal < 0;
-            for (int i = lane; i < C * NW; i += 32) {
-                const int c = i / NW, w = i - c * NW;
-                uint32_t d = S.planes[c * NWP + w].x;
-                const uint32_t st = S.setp[i], cl = S.clrp[i];
-                if (st | cl) {
-                    S.setp[i] = 0u;
-                    S.clrp[i] = 0u;
-                    d = (d & ~cl) | (~d & st);
-                    put_word(S.planes, NWP, c, w, d);
-                }
-                if (c == cf.ch_goal)
-                    gl |= d != 0u;
-            }
-            goal_left = __any_sync(0xffffffffu, gl);
-            done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
-            if (done && cf.auto_reset) {
-                for (int i = lane; i < C * NW; i += 32) {
-                    const int c = i / NW, w = i - c * NW;
-                    put_word(S.planes, NWP, c, w, S.basep[i]);
-                }
-                t = 0;
-                gl = cf.ch_goal < 0;
-                if (cf.ch_goal >= 0)
-                    for (int w = lane; w < NW; w += 32)
-                        gl |= S.basep[cf.ch_goal * NW + w] != 0u;
-                goal_left = __any_sync(0xffffffffu, gl);
-            }
-            __syncwarp();  // the new board
-            force_planes(cf, S.planes, S.masks, 0, 1, C + 1);
-            __syncwarp();  // its force planes
+            const int3 r = env_board_update(cf, S.planes, S.setp, S.clrp, S.basep, S.masks, t);
+            t = r.x;
+            goal_left = r.y;
+            done = r.z;
             f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
             sum += rew;
         }
@@ -1819,22 +1878,11 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
         if (lane < NW)
             slot[lane] = f_next;
         __syncwarp();
-        if (traj && lane == 0) {
-            if (rew_traj)
-                rew_traj[(size_t)s * cf.B + env] = rew;
-            if (done_traj)
-                done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
-        }
-        if (obs_traj) {
-            CellT *dst = obs_traj + ((size_t)s * cf.B + env) * HW;
-            for (int p = lane; p < HW; p += 32)
-                dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
-        }
+        if (any_traj)
+            env_step_outputs<CellT>(cf, S.planes, env, s, rew, done, obs_traj, rew_traj, done_traj);
         ++s;
     }
-    CellT *dst = cur + (size_t)env * HW;
-    for (int p = lane; p < HW; p += 32)
-        dst[p] = (CellT)gather_cell(cf, S.planes, nullptr, p);
+    store_cells<CellT>(cf, S.planes, cur + (size_t)env * HW, lane, 32);
     if (lane == 0) {
         tsteps[env] = t;
         if (rew_sum)
