@@ -292,6 +292,15 @@ void compile_table(const av_rule *rules, const DevConfig &cf, const double *dens
         hd[2] = no;
         n_outs += no;
     }
+    // one batch of passing terms after the last rule's: a read one batch past
+    // any rule's terms stays inside the term list
+    for (int j = 0; j < kRestBatch; ++j) {
+        for (int g = 0; g < 4; ++g) {
+            terms.push_back((uint32_t)((cf.C + 1) * cf.NWP * 8));
+            terms.push_back(kTermAbsent);
+        }
+        ++n_terms;
+    }
     const uint32_t tw = table_terms_word(R), ow = table_outs_word(R, n_terms);
     arena.resize(base + ow + outs.size(), 0);
     uint32_t *t = &arena[base];

@@ -31,7 +31,8 @@
 //           (byte offset of plane entry c*NWP + (s >> 5), s & 31 | kTermAbsent
 //           for an absent term; funnel shifts use only the low five bits);
 //           each rule's list is followed by padding terms up to a whole
-//           number of kRestBatch terms after its first kRegTerms present ones
+//           number of kRestBatch terms after its first kRegTerms present ones,
+//           and the table's list ends with one more batch of padding terms
 //   outputs (uint4, [output][rotation]): (s >> 5, s & 31, set bits, clear bits)
 #pragma once
 
@@ -1507,22 +1508,19 @@ __device__ __forceinline__ int2 env_rule_rest(const DevConfig &cf, const uint32_
     const uint32_t t0 = min(h0.x, (uint32_t)kRegTerms);
     const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)(h1.x + t0) * 4 + g;
     const uint32_t nb = (h0.x + h0.y - t0 + kRestBatch - 1) / kRestBatch;  // padded batches
+    // the table ends its term list with a batch of passing terms, so a batch
+    // read past this rule's last one stays inside the list
     uint2 dn[kRestBatch];
-    if (nb > 0) {
 #pragma unroll
-        for (int j = 0; j < kRestBatch; ++j)
-            dn[j] = ld2<SM>(tp + 4 * j);
-    }
+    for (int j = 0; j < kRestBatch; ++j)
+        dn[j] = ld2<SM>(tp + 4 * j);
     for (uint32_t b = 0; b < nb; ++b) {
         uint2 d[kRestBatch];
+        tp += 4 * kRestBatch;
 #pragma unroll
-        for (int j = 0; j < kRestBatch; ++j)
+        for (int j = 0; j < kRestBatch; ++j) {
             d[j] = dn[j];
-        if (b + 1 < nb) {
-            tp += 4 * kRestBatch;
-#pragma unroll
-            for (int j = 0; j < kRestBatch; ++j)
-                dn[j] = ld2<SM>(tp + 4 * j);
+            dn[j] = ld2<SM>(tp + 4 * j);
         }
 #pragma unroll
         for (int u = 0; u < NA; ++u) {
@@ -1766,14 +1764,15 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
 
     int sum = 0;
     uint32_t m[RPW][NA];  // anchors of each rule live after its register terms
-    // Steps in which no rule survives its register terms: t advances, the next
-    // step's force goes into the slot, nothing else changes.  The loop is kept
-    // free of branches around rarely used code, which cost tens of cycles each
-    // even when not taken.  Returns true when step s has a live rule (its masks
-    // left in m for the general step).
-    auto quiet_steps = [&](int &s, int lim, auto traj_tag) -> bool {
+    // Steps in which no rule survives its register terms and no reset is due:
+    // t advances, the next step's force goes into the slot, nothing else
+    // changes.  The loop is kept free of branches around rarely used code,
+    // which cost tens of cycles each even when not taken.  Leaves s at the
+    // first step it does not finish (lim at the latest), with that step's
+    // register masks in m when s < lim.
+    auto quiet_steps = [&](int &s, int lim, auto traj_tag) {
         constexpr bool TRAJ = decltype(traj_tag)::value;
-        while (s < lim && (!cf.auto_reset || (goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps)))) {
+        while (s < lim) {
             const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
             const uint2 f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
             uint32_t anyall = 0;
@@ -1784,8 +1783,9 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
                     m[k][u] = env_reg_terms(fr[k], u);
                     anyall |= m[k][u];
                 }
-            if (__any_sync(0xffffffffu, anyall != 0u))
-                return true;  // the general step takes it
+            const bool reset_due = cf.auto_reset && !(goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps));
+            if (__any_sync(0xffffffffu, anyall != 0u) || reset_due)
+                return;  // the general step takes it
             t += 1;
             if (TRAJ) {
                 const int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
@@ -1803,7 +1803,6 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
             __syncwarp();
             ++s;
         }
-        return false;
     };
     const bool any_traj = traj || obs_traj != nullptr;
     int refilled = 0;
@@ -1815,17 +1814,12 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
             refilled = s;
         }
         const int lim = min(n_steps, ((s / (kActChunk / 2)) + 1) * (kActChunk / 2));
-        const bool live_rule = any_traj ? quiet_steps(s, lim, std::integral_constant<bool, true>())
-                                        : quiet_steps(s, lim, std::integral_constant<bool, false>());
+        if (any_traj)
+            quiet_steps(s, lim, std::integral_constant<bool, true>());
+        else
+            quiet_steps(s, lim, std::integral_constant<bool, false>());
         if (s >= lim)
             continue;  // the end, or the next refill
-        if (!live_rule) {  // a reset is due: no register masks yet
-#pragma unroll
-            for (int k = 0; k < RPW; ++k)
-#pragma unroll
-                for (int u = 0; u < NA; ++u)
-                    m[k][u] = env_reg_terms(fr[k], u);
-        }
 
         // ---- general step s: the rest of every live rule, writes
         const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
