@@ -1821,60 +1821,78 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
         if (s >= lim)
             continue;  // the end, or the next refill
 
-        // ---- general step s: the rest of every live rule, writes
-        const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
-        uint2 f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
-        uint32_t bits = 0;
+        // ---- busy steps: while some rule passes its register terms (or a
+        // reset is due) every step is a general step; their own loop, so that
+        // a run of them does not leave and re-enter the quiet loop each step.
+        // The first recomputes what the quiet loop stopped at.
+        while (s < lim) {
+            const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
+            uint2 f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
+            uint32_t anyall = 0;
 #pragma unroll
-        for (int k = 0; k < RPW; ++k) {
-            uint32_t a = 0;
+            for (int k = 0; k < RPW; ++k)
 #pragma unroll
-            for (int u = 0; u < NA; ++u)
-                a |= m[k][u];
-            bits |= (a != 0u ? 1u : 0u) << k;
-        }
-        int rew = 0, changed = 0;
-        {
-            uint32_t live = __reduce_or_sync(0xffffffffu, bits);
-            int2 acc = make_int2(0, 0);
-            while (live) {
-                const int k = __ffs(live) - 1;
-                live &= live - 1;
-                uint32_t mk[NA];
+                for (int u = 0; u < NA; ++u) {
+                    m[k][u] = env_reg_terms(fr[k], u);
+                    anyall |= m[k][u];
+                }
+            const bool reset_due = cf.auto_reset && !(goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps));
+            if (!__any_sync(0xffffffffu, anyall != 0u) && !reset_due)
+                break;  // a quiet step: back to the quiet loop
+
+            // ---- general step s: the rest of every live rule, writes
+            uint32_t bits = 0;
+#pragma unroll
+            for (int k = 0; k < RPW; ++k) {
+                uint32_t a = 0;
 #pragma unroll
                 for (int u = 0; u < NA; ++u)
-                    mk[u] = 0;
-#pragma unroll
-                for (int kk = 0; kk < RPW; ++kk)
-                    if (kk == k)
-#pragma unroll
-                        for (int u = 0; u < NA; ++u)
-                            mk[u] = m[kk][u];
-                const int2 o = env_rule_rest<NA, SM>(cf, tab, pbase, S.setp, S.clrp, k, mk);
-                acc.x += o.x;
-                acc.y |= o.y;
+                    a |= m[k][u];
+                bits |= (a != 0u ? 1u : 0u) << k;
             }
-            rew = __reduce_add_sync(0xffffffffu, acc.x);
-            changed = __any_sync(0xffffffffu, acc.y != 0);
-        }
+            int rew = 0, changed = 0;
+            {
+                uint32_t live = __reduce_or_sync(0xffffffffu, bits);
+                int2 acc = make_int2(0, 0);
+                while (live) {
+                    const int k = __ffs(live) - 1;
+                    live &= live - 1;
+                    uint32_t mk[NA];
+#pragma unroll
+                    for (int u = 0; u < NA; ++u)
+                        mk[u] = 0;
+#pragma unroll
+                    for (int kk = 0; kk < RPW; ++kk)
+                        if (kk == k)
+#pragma unroll
+                            for (int u = 0; u < NA; ++u)
+                                mk[u] = m[kk][u];
+                    const int2 o = env_rule_rest<NA, SM>(cf, tab, pbase, S.setp, S.clrp, k, mk);
+                    acc.x += o.x;
+                    acc.y |= o.y;
+                }
+                rew = __reduce_add_sync(0xffffffffu, acc.x);
+                changed = __any_sync(0xffffffffu, acc.y != 0);
+            }
 
-        t += 1;
-        int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
-        if (changed || (done && cf.auto_reset)) {
-            const int3 r = env_board_update(cf, S.planes, S.setp, S.clrp, S.basep, S.masks, t);
-            t = r.x;
-            goal_left = r.y;
-            done = r.z;
-            f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
-            sum += rew;
+            t += 1;
+            int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+            if (changed || (done && cf.auto_reset)) {
+                const int3 r = env_board_update(cf, S.planes, S.setp, S.clrp, S.basep, S.masks, t);
+                t = r.x;
+                goal_left = r.y;
+                done = r.z;
+                f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
+                sum += rew;
+            }
+            // every read of this step's force is behind the step's last vote
+            if (lane < NW)
+                slot[lane] = f_next;
+            __syncwarp();
+            if (any_traj)
+                env_step_outputs<CellT>(cf, S.planes, env, s, rew, done, obs_traj, rew_traj, done_traj);
+            ++s;
         }
-        // every read of this step's force is behind the step's last vote
-        if (lane < NW)
-            slot[lane] = f_next;
-        __syncwarp();
-        if (any_traj)
-            env_step_outputs<CellT>(cf, S.planes, env, s, rew, done, obs_traj, rew_traj, done_traj);
-        ++s;
     }
     store_cells<CellT>(cf, S.planes, cur + (size_t)env * HW, lane, 32);
     if (lane == 0) {
