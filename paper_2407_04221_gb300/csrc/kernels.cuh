@@ -1475,6 +1475,7 @@ template <int NA>
 struct EnvRule {
     uint32_t vm[NA];
     uint32_t a[kRegTerms], s[kRegTerms];
+    uint32_t rest;  // the remaining terms: (first descriptor index for this lane's rotation) << 8 | batches
 };
 
 // Anchors of this lane's word u that pass the register-resident terms.
@@ -1491,8 +1492,9 @@ __device__ __forceinline__ uint32_t env_reg_terms(const EnvRule<NA> &f, int u)
 }
 
 // The terms of rule r after its register-resident ones, for one environment,
-// then the rule's write.  `m` holds the anchors live after the register terms;
-// `pbase` is the shared address of this lane's word in plane 0.  Every
+// then the rule's write.  `rest` locates those terms (EnvRule::rest); `m`
+// holds the anchors live after the register terms; `pbase` is the shared
+// address of this lane's word in plane 0.  Every
 // remaining term is evaluated, kRestBatch per iteration (the padded list has
 // whole batches) with the next batch's descriptors already loaded: a rule that
 // gets this far usually has few live anchors, and a warp vote per few terms
@@ -1500,14 +1502,12 @@ __device__ __forceinline__ uint32_t env_reg_terms(const EnvRule<NA> &f, int u)
 // this lane matched).
 template <int NA, bool SM>
 __device__ __forceinline__ int2 env_rule_rest(const DevConfig &cf, const uint32_t *tab, uint32_t pbase,
-                                              uint32_t *setp, uint32_t *clrp, int r, uint32_t (&m)[NA])
+                                              uint32_t *setp, uint32_t *clrp, int r, uint32_t rest,
+                                              uint32_t (&m)[NA])
 {
     const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
-    const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
-    const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
-    const uint32_t t0 = min(h0.x, (uint32_t)kRegTerms);
-    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)(h1.x + t0) * 4 + g;
-    const uint32_t nb = (h0.x + h0.y - t0 + kRestBatch - 1) / kRestBatch;  // padded batches
+    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (rest >> 8);
+    const uint32_t nb = rest & 0xffu;  // padded batches
     // the table ends its term list with a batch of passing terms, so a batch
     // read past this rule's last one stays inside the list
     uint2 dn[kRestBatch];
@@ -1544,6 +1544,8 @@ __device__ __forceinline__ int2 env_rule_rest(const DevConfig &cf, const uint32_
         cnt += __popc(m[u]);
     if (cnt == 0)
         return make_int2(0, 0);
+    const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
+    const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
     const uint4 *op = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, tab[1])) + (size_t)h1.y * 4 + g;
     for (uint32_t o = 0; o < h0.z; ++o) {
         const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
@@ -1731,6 +1733,7 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
                 f.a[j] = pbase + ones;
                 f.s[j] = 0;
             }
+            f.rest = 0;
             if (k < cf.R) {
                 const uint4 h0 = ld4<SM>(tab + 4 + 8 * k);
                 const uint4 h1 = ld4<SM>(tab + 8 + 8 * k);
@@ -1747,6 +1750,9 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
                         f.a[j] = pbase + d.x;
                         f.s[j] = d.y;
                     }
+                const uint32_t t0 = min(h0.x, (uint32_t)kRegTerms);
+                const uint32_t nb = (h0.x + h0.y - t0 + kRestBatch - 1) / kRestBatch;  // padded batches
+                f.rest = (((h1.x + t0) * 4 + g) << 8) | nb;
             }
         }
     }
@@ -1828,46 +1834,42 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
         while (s < lim) {
             const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
             uint2 f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
-            uint32_t anyall = 0;
-#pragma unroll
-            for (int k = 0; k < RPW; ++k)
-#pragma unroll
-                for (int u = 0; u < NA; ++u) {
-                    m[k][u] = env_reg_terms(fr[k], u);
-                    anyall |= m[k][u];
-                }
-            const bool reset_due = cf.auto_reset && !(goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps));
-            if (!__any_sync(0xffffffffu, anyall != 0u) && !reset_due)
-                break;  // a quiet step: back to the quiet loop
-
-            // ---- general step s: the rest of every live rule, writes
             uint32_t bits = 0;
 #pragma unroll
             for (int k = 0; k < RPW; ++k) {
                 uint32_t a = 0;
 #pragma unroll
-                for (int u = 0; u < NA; ++u)
+                for (int u = 0; u < NA; ++u) {
+                    m[k][u] = env_reg_terms(fr[k], u);
                     a |= m[k][u];
+                }
                 bits |= (a != 0u ? 1u : 0u) << k;
             }
+            uint32_t live = __reduce_or_sync(0xffffffffu, bits);  // rules live past their register terms
+            const bool reset_due = cf.auto_reset && !(goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps));
+            if (!live && !reset_due)
+                break;  // a quiet step: back to the quiet loop
+
+            // ---- general step s: the rest of every live rule, writes
             int rew = 0, changed = 0;
             {
-                uint32_t live = __reduce_or_sync(0xffffffffu, bits);
                 int2 acc = make_int2(0, 0);
                 while (live) {
                     const int k = __ffs(live) - 1;
                     live &= live - 1;
-                    uint32_t mk[NA];
+                    uint32_t mk[NA], rk = 0;
 #pragma unroll
                     for (int u = 0; u < NA; ++u)
                         mk[u] = 0;
 #pragma unroll
                     for (int kk = 0; kk < RPW; ++kk)
-                        if (kk == k)
+                        if (kk == k) {
 #pragma unroll
                             for (int u = 0; u < NA; ++u)
                                 mk[u] = m[kk][u];
-                    const int2 o = env_rule_rest<NA, SM>(cf, tab, pbase, S.setp, S.clrp, k, mk);
+                            rk = fr[kk].rest;
+                        }
+                    const int2 o = env_rule_rest<NA, SM>(cf, tab, pbase, S.setp, S.clrp, k, rk, mk);
                     acc.x += o.x;
                     acc.y |= o.y;
                 }
