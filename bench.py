@@ -168,6 +168,19 @@ def valid_anchor_rules(wl: wk.Workload, rules: np.ndarray) -> float:
     return float((2 * va + 2 * vb).sum(-1).mean())
 
 
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The largest x over the ranks of the default process group (x itself
+    with one rank).  `device` is where the reduction runs: the rank's GPU
+    under NCCL, the CPU under gloo."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -338,11 +351,7 @@ def run_ours(args, wl):
     ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
     kernel_ms = sum(ms) / len(ms)
     total_ms = sum(ms)
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(total_ms, world, dev)
     env_steps = wl.batch * wl.steps * args.steps * world
     value = env_steps / (total_ms / 1e3)
 
@@ -363,11 +372,7 @@ def run_ours(args, wl):
     e1.record(stream)
     barrier()
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
     e2e_value = wl.batch * wl.steps * world / (e2e_ms / 1e3)
 
     if rank == 0:
@@ -487,11 +492,7 @@ def run_search(args, wl):
     clocks = sampler.stop()
     env.sync()
     total_ms = sum(a.elapsed_time(b) for a, b in zip(starts, ends))
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(total_ms, world, dev)
     value = children * args.steps * world / (total_ms / 1e3)
 
     # ---- the expand kernel alone: events around each av_expand of one search
@@ -543,7 +544,7 @@ def run_search(args, wl):
         host_best.copy_(r["trace_best"], non_blocking=True)
     e1.record(stream)
     barrier()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
     e2e_value = children * world / (e2e_ms / 1e3)
 
     if rank == 0:
