@@ -277,7 +277,10 @@ def run_reference(args, wl):
 
 
 def config_dict(wl, sample=None):
-    d = {"workload": f"{wl.name} (BASELINE config {wl.key})", "batch": wl.batch, "H": wl.H,
+    full = wk.WORKLOADS[wl.key]
+    name = wl.name if (wl.batch, wl.steps) == (full.batch, full.steps) else \
+        f"{wl.name}, smaller case: {wl.batch} envs x {wl.steps} steps"
+    d = {"workload": name, "batch": wl.batch, "H": wl.H,
          "W": wl.W, "tile_channels": wl.C, "rules": wl.n_rules, "rotations": 4,
          "pattern_sizes": [f"{h}x{w}" for h, w in wl.shapes],
          "fused_steps_per_launch": wl.steps, "per_env_rules": bool(wl.rules_per_env),
@@ -674,6 +677,10 @@ def main(argv=None):
     ap.add_argument("--config", type=int, default=2, choices=(2, 3, 4, 5))
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="run a smaller case of the workload (profiling): this many envs")
+    ap.add_argument("--fused-steps", type=int, default=0,
+                    help="run a smaller case of the workload (profiling): steps per launch")
     ap.add_argument("--int-probe", action="store_true", help="measure integer issue rate and exit")
     args = ap.parse_args(argv)
     if args.int_probe:
@@ -681,6 +688,10 @@ def main(argv=None):
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     wl = workload_for(args.config)
+    if args.batch > 0:
+        wl = wl.scaled(batch=args.batch)
+    if args.fused_steps > 0 and not wl.frontier:
+        wl = wl.scaled(steps=args.fused_steps)
     if wl.frontier:
         return run_search_reference(args, wl) if args.impl == "reference" else run_search(args, wl)
     if args.impl == "reference":
