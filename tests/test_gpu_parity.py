@@ -270,3 +270,35 @@ def test_both_kernel_paths_edges(monkeypatch, path, H, W, C, shapes, R):
     np.testing.assert_array_equal(to_np(res["rew"]), ref["rew"])
     np.testing.assert_array_equal(to_np(res["done"]), ref["done"])
     env.close()
+
+
+# ------------------------------------- launch lengths around the action ring
+@pytest.mark.parametrize("path", ["block", "fast", "warp"])
+def test_launch_lengths_and_continuation(monkeypatch, path):
+    """Rollouts of 0 and 1 steps, lengths around the 128-step refill of the
+    pre-drawn actions, and launches that continue one another, each compared
+    with the oracle run for the total length (trajectories and auto-reset on,
+    so resets fall inside and across launches)."""
+    import paper_2407_04221_gb300 as av
+    monkeypatch.setenv("AV_KERNEL_PATH", path)
+    wl = wk.WORKLOADS[3].scaled(batch=6, max_steps=37)
+    env, cfg, rules, cum = make(wl, 31)
+    assert av.av_rollout_path(env.h) == _PATH_IDS[path]
+    s = wk.seeds(31)
+    g0 = to_np(env.reset(s["reset"]))
+    ids = np.arange(wl.batch)
+    lengths = [0, 1, 127, 128, 129, 255, 257]
+    t0 = np.zeros(wl.batch, np.int32)
+    g = g0
+    for n, seed in zip(lengths, range(900, 900 + len(lengths))):
+        res = env.rollout(n, seed, trajectory=True)
+        ref = oracle.rollout(cfg, rules, g, g0, t0, n, seed, env_ids=ids, trajectory=True)
+        if n:
+            np.testing.assert_array_equal(to_np(res["obs"]), ref["obs"])
+            np.testing.assert_array_equal(to_np(res["rew"]), ref["rew"])
+            np.testing.assert_array_equal(to_np(res["done"]), ref["done"])
+        got, t = env.get_state()
+        np.testing.assert_array_equal(to_np(got), ref["grids"])
+        np.testing.assert_array_equal(to_np(t), ref["t"])
+        g, t0 = ref["grids"], ref["t"]
+    env.close()
