@@ -35,7 +35,7 @@ void block_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off
                                                                    (CellT *)children, rewards, done, hashes);
 }
 
-template <typename CellT, int NA, int RB>
+template <typename CellT, int NA>
 void warp_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
             const uint32_t *masks, const void *parents, int F, const int32_t *n_parent, void *children,
             int32_t *rewards, uint8_t *done, uint64_t *hashes, cudaStream_t st)
@@ -46,11 +46,11 @@ void warp_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
     const ExpandLayout L = expand_layout(cf);
     const size_t sm = L.warps + (size_t)wpc * L.per_warp;
     if (cf.rule_words > 0)
-        expand_warp_kernel<CellT, NA, RB, true><<<grid, 32 * wpc, sm, st>>>(
+        expand_warp_kernel<CellT, NA, true><<<grid, 32 * wpc, sm, st>>>(
             cf, arena, tab_off, vm, masks, (const CellT *)parents, F, n_parent, (CellT *)children, rewards,
             done, hashes);
     else
-        expand_warp_kernel<CellT, NA, RB, false><<<grid, 32 * wpc, sm, st>>>(
+        expand_warp_kernel<CellT, NA, false><<<grid, 32 * wpc, sm, st>>>(
             cf, arena, tab_off, vm, masks, (const CellT *)parents, F, n_parent, (CellT *)children, rewards,
             done, hashes);
 }
@@ -70,13 +70,13 @@ cudaError_t configure_expand()
     AV_FOR_NA(AV_SET, uint8_t)
     AV_FOR_NA(AV_SET, uint16_t)
 #undef AV_SET
-#define AV_SETW(CELL, NA, RB)                                            \
-    set((const void *)expand_warp_kernel<CELL, NA, RB, true>);           \
-    set((const void *)expand_warp_kernel<CELL, NA, RB, false>);
-    AV_SETW(uint8_t, 1, 4)
-    AV_SETW(uint8_t, 2, 2)
-    AV_SETW(uint16_t, 1, 4)
-    AV_SETW(uint16_t, 2, 2)
+#define AV_SETW(CELL, NA)                                            \
+    set((const void *)expand_warp_kernel<CELL, NA, true>);           \
+    set((const void *)expand_warp_kernel<CELL, NA, false>);
+    AV_SETW(uint8_t, 1)
+    AV_SETW(uint8_t, 2)
+    AV_SETW(uint16_t, 1)
+    AV_SETW(uint16_t, 2)
 #undef AV_SETW
     return e;
 }
@@ -89,17 +89,17 @@ void launch_expand(const DevConfig &cf, const uint32_t *arena, const uint32_t *t
     if (use_warp_expand(cf)) {
         if (cf.NA == 1) {
             if (u8)
-                warp_t<uint8_t, 1, 4>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards, done,
+                warp_t<uint8_t, 1>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards, done,
                                       hashes, st);
             else
-                warp_t<uint16_t, 1, 4>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards,
+                warp_t<uint16_t, 1>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards,
                                        done, hashes, st);
         } else {
             if (u8)
-                warp_t<uint8_t, 2, 2>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards, done,
+                warp_t<uint8_t, 2>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards, done,
                                       hashes, st);
             else
-                warp_t<uint16_t, 2, 2>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards,
+                warp_t<uint16_t, 2>(cf, arena, tab_off, vm, masks, parents, F, n_parent, children, rewards,
                                        done, hashes, st);
         }
         return;

@@ -199,6 +199,14 @@ __device__ __forceinline__ uint2 ld2(const uint2 *p)
 }
 
 // Write plane word w of channel c into the doubled layout.
+// 64-bit shared load from a shared-window address.
+__device__ __forceinline__ uint2 lds2(uint32_t addr)
+{
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
 __device__ __forceinline__ void put_word(uint2 *planes, int NWP, int c, int w, uint32_t v)
 {
     planes[c * NWP + w].x = v;
@@ -313,6 +321,43 @@ __device__ __forceinline__ void write_force(const DevConfig &cf, const Smem &S, 
 {
     force_plane(cf, S.planes, S.masks, action);
 }
+
+// Force planes of actions a0, a0 + stride, ... < 5 from the player plane (one
+// warp), into planes first + action.
+static __device__ void force_planes(const DevConfig &cf, uint2 *P, const uint32_t *masks, int a0, int stride,
+                                    int first)
+{
+    const int lane = threadIdx.x & 31, NW = cf.NW, NWP = cf.NWP;
+    const uint32_t *firstcol = masks, *lastcol = masks + NW, *cellmask = masks + 2 * NW;
+    const uint2 *pl = P + (cf.ch_player >= 0 ? cf.ch_player : 0) * NWP;
+    for (int action = a0; action < 5; action += stride)
+        for (int w = lane; w < NW; w += 32) {
+            uint32_t f = 0;
+            if (cf.ch_player >= 0 && action > 0) {
+                const int n = (action == 1 || action == 3) ? cf.W : 1;
+                const int q = n >> 5, r = n & 31;
+                if (action == 1 || action == 4) {
+                    const uint2 e = pl[w + q];
+                    f = __funnelshift_r(e.x, e.y, r);
+                } else {
+                    const int j = w - q;
+                    if (j >= 1) {
+                        const uint2 e = pl[j - 1];
+                        f = __funnelshift_l(e.x, e.y, r);
+                    } else if (j == 0) {
+                        f = pl[0].x << r;
+                    }
+                }
+                if (action == 2)
+                    f &= ~firstcol[w];
+                else if (action == 4)
+                    f &= ~lastcol[w];
+                f &= cellmask[w];
+            }
+            put_word(P, NWP, first + action, w, f);
+        }
+}
+
 
 __device__ __forceinline__ void scatter_bits(uint32_t *dst, uint32_t chans, int NW, int w0, uint32_t lo,
                                              uint32_t hi)
@@ -612,74 +657,12 @@ expand_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *
 
 constexpr int kWarpCtaMax = 8;  // warps (= parents) per CTA at most
 
-struct WarpLayout {
-    size_t planes, setp, clrp, basep, vm, masks, acts, rules, cells, total;
-};
-
-__host__ __device__ inline WarpLayout warp_layout(const DevConfig &cf, int n_cell_boards)
-{
-    WarpLayout L;
-    const size_t pw = (size_t)cf.C * cf.NW * 4;
-    L.planes = 0;
-    L.setp = align16((size_t)(cf.C + 1) * cf.NWP * 8);
-    L.clrp = align16(L.setp + pw);
-    L.basep = align16(L.clrp + pw);
-    L.vm = align16(L.basep + pw);
-    L.masks = align16(L.vm + (size_t)kShapes * cf.NW * 4);
-    L.acts = align16(L.masks + (size_t)3 * cf.NW * 4);
-    L.rules = align16(L.acts + kActChunk);
-    L.cells = align16(L.rules + (size_t)cf.rule_words * 4);
-    L.total = align16(L.cells + (size_t)n_cell_boards * cf.HW * 2);
-    return L;
-}
-
 struct WarpSmem {
     uint2 *planes;
     uint32_t *setp, *clrp, *basep, *vm, *masks, *rules;
     uint8_t *acts;
     uint16_t *cells;
 };
-
-__device__ __forceinline__ WarpSmem carve_warp(unsigned char *smem, const DevConfig &cf, int n_cell_boards)
-{
-    const WarpLayout L = warp_layout(cf, n_cell_boards);
-    unsigned char *b = smem + (size_t)(threadIdx.x >> 5) * L.total;
-    WarpSmem m;
-    m.planes = reinterpret_cast<uint2 *>(b + L.planes);
-    m.setp = reinterpret_cast<uint32_t *>(b + L.setp);
-    m.clrp = reinterpret_cast<uint32_t *>(b + L.clrp);
-    m.basep = reinterpret_cast<uint32_t *>(b + L.basep);
-    m.vm = reinterpret_cast<uint32_t *>(b + L.vm);
-    m.masks = reinterpret_cast<uint32_t *>(b + L.masks);
-    m.acts = b + L.acts;
-    m.rules = reinterpret_cast<uint32_t *>(b + L.rules);
-    m.cells = reinterpret_cast<uint16_t *>(b + L.cells);
-    return m;
-}
-
-static __device__ void warp_stage(const DevConfig &cf, const WarpSmem &S, const uint32_t *__restrict__ vm_g,
-                           const uint32_t *__restrict__ masks_g, const uint32_t *__restrict__ tab_g,
-                           uint32_t tab_words, bool rules_to_smem)
-{
-    const int lane = threadIdx.x & 31;
-    for (int i = lane; i < (cf.C + 1) * cf.NWP; i += 32)
-        S.planes[i] = make_uint2(0u, 0u);
-    for (int i = lane; i < cf.C * cf.NW; i += 32) {
-        S.setp[i] = 0u;
-        S.clrp[i] = 0u;
-    }
-    for (int i = lane; i < kShapes * cf.NW; i += 32)
-        S.vm[i] = __ldg(vm_g + i);
-    for (int i = lane; i < 3 * cf.NW; i += 32)
-        S.masks[i] = __ldg(masks_g + i);
-    if (rules_to_smem) {
-        const uint4 *src = reinterpret_cast<const uint4 *>(tab_g);
-        uint4 *d = reinterpret_cast<uint4 *>(S.rules);
-        for (uint32_t i = lane; i < tab_words / 4; i += 32)
-            d[i] = __ldg(src + i);
-    }
-    __syncwarp();
-}
 
 template <typename CellT>
 __device__ void warp_cells_to_planes(const DevConfig &cf, const CellT *__restrict__ src, uint2 *dbl,
@@ -702,153 +685,6 @@ __device__ void warp_cells_to_planes(const DevConfig &cf, const CellT *__restric
     }
 }
 
-template <int NA>
-struct Words {
-    uint32_t v[NA];
-};
-
-// Remaining terms of a rule that survived its first two, then its write.
-// Returns (this lane's reward, 1 if this lane wrote an output).
-template <int NA, bool SM>
-__device__ __noinline__ int2 warp_rule_rest(const DevConfig &cf, const uint32_t *tab, const WarpSmem &S, int r,
-                                            Words<NA> mw)
-{
-    uint32_t *m = mw.v;
-    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
-    const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
-    const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
-    const uint2 *tp = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R)) + (size_t)h1.x * 4 + g;
-    const unsigned char *pb = reinterpret_cast<const unsigned char *>(S.planes) + q * 8;
-    const uint32_t np = h0.x, nt = h0.x + h0.y;
-    for (uint32_t t = 2; t < nt; t += 2) {
-        const bool two = t + 1 < nt && (t + 1 < np || t >= np);
-        const uint32_t neg = t < np ? 0u : 0xffffffffu;
-        const uint2 d0 = ld2<SM>(tp + 4 * t);
-        const uint2 d1 = two ? ld2<SM>(tp + 4 * t + 4) : d0;
-        uint32_t any = 0;
-#pragma unroll
-        for (int u = 0; u < NA; ++u) {
-            const uint2 w0 = *reinterpret_cast<const uint2 *>(pb + d0.x + 64 * u);
-            const uint2 w1 = *reinterpret_cast<const uint2 *>(pb + d1.x + 64 * u);
-            m[u] &= (__funnelshift_r(w0.x, w0.y, d0.y) ^ neg) & (__funnelshift_r(w1.x, w1.y, d1.y) ^ neg);
-            any |= m[u];
-        }
-        if (!two)
-            t -= 1;
-        if (!__any_sync(0xffffffffu, any != 0u))
-            return make_int2(0, 0);
-    }
-    uint32_t cnt = 0;
-#pragma unroll
-    for (int u = 0; u < NA; ++u)
-        cnt += __popc(m[u]);
-    if (cnt == 0)
-        return make_int2(0, 0);
-    const uint4 *op = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, tab[1])) + (size_t)h1.y * 4 + g;
-    for (uint32_t o = 0; o < h0.z; ++o) {
-        const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
-#pragma unroll
-        for (int u = 0; u < NA; ++u) {
-            if (!m[u])
-                continue;
-            const int w0 = q + 8 * u + (int)ov.x;
-            const uint32_t lo = m[u] << ov.y;
-            const uint32_t hi = ov.y ? (m[u] >> (32u - ov.y)) : 0u;
-            scatter_bits(S.setp, ov.z, cf.NW, w0, lo, hi);
-            scatter_bits(S.clrp, ov.w, cf.NW, w0, lo, hi);
-        }
-    }
-    return make_int2((int)h0.w * (int)cnt, 1);
-}
-
-// Every rule of the env against the warp's planes.  The first two terms of RB
-// rules are evaluated without branches (independent chains the scheduler can
-// overlap); one warp reduction yields the rules that still have a live anchor.
-// Returns (this lane's reward, 1 if this lane wrote an output).
-template <int NA, int RB, bool SM>
-__device__ __forceinline__ int2 warp_rules(const DevConfig &cf, const uint32_t *tab, const WarpSmem &S)
-{
-    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
-    const unsigned char *pb = reinterpret_cast<const unsigned char *>(S.planes) + q * 8;
-    const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
-    const uint32_t total_terms = tab[1];
-    int2 acc = make_int2(0, 0);
-    for (int r0 = 0; r0 < cf.R; r0 += RB) {
-        uint32_t m[RB][NA];
-        uint32_t live = 0;
-#pragma unroll
-        for (int j = 0; j < RB; ++j) {
-            const bool ok = r0 + j < cf.R;
-            const int r = ok ? r0 + j : 0;
-            const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
-            const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
-            const uint32_t *vmr = S.vm + ((h1.z >> (8 * g)) & 0xffu) * cf.NW;
-            const uint32_t np = h0.x, nt = ok ? h0.x + h0.y : 0u;
-            // descriptors of terms 0 and 1 (index clamped to a valid term)
-            const uint32_t t0 = nt > 0 ? h1.x : 0u, t1 = nt > 1 ? h1.x + 1 : t0;
-            const uint2 d0 = total_terms ? ld2<SM>(terms + (size_t)t0 * 4 + g) : make_uint2(0u, 0u);
-            const uint2 d1 = total_terms ? ld2<SM>(terms + (size_t)t1 * 4 + g) : make_uint2(0u, 0u);
-            const uint32_t keep0 = nt > 0 ? 0u : 0xffffffffu;  // no term: pass every anchor
-            const uint32_t keep1 = nt > 1 ? 0u : 0xffffffffu;
-            const uint32_t neg0 = np > 0 ? 0u : 0xffffffffu;
-            const uint32_t neg1 = np > 1 ? 0u : 0xffffffffu;
-            uint32_t any = 0;
-#pragma unroll
-            for (int u = 0; u < NA; ++u) {
-                const int a = q + 8 * u;
-                const uint2 w0 = *reinterpret_cast<const uint2 *>(pb + d0.x + 64 * u);
-                const uint2 w1 = *reinterpret_cast<const uint2 *>(pb + d1.x + 64 * u);
-                const uint32_t x0 = (__funnelshift_r(w0.x, w0.y, d0.y) ^ neg0) | keep0;
-                const uint32_t x1 = (__funnelshift_r(w1.x, w1.y, d1.y) ^ neg1) | keep1;
-                const uint32_t v = (ok && a < cf.NW) ? vmr[a] : 0u;
-                m[j][u] = v & x0 & x1;
-                any |= m[j][u];
-            }
-            live |= (any != 0u ? 1u : 0u) << j;
-        }
-        live = __reduce_or_sync(0xffffffffu, live);
-        while (live) {  // rare: rules with a live anchor after two terms
-            const int j = __ffs(live) - 1;
-            live &= live - 1;
-            Words<NA> mw;
-#pragma unroll
-            for (int jj = 0; jj < RB; ++jj)
-                if (jj == j)
-#pragma unroll
-                    for (int u = 0; u < NA; ++u)
-                        mw.v[u] = m[jj][u];
-            const int2 o = warp_rule_rest<NA, SM>(cf, tab, S, r0 + j, mw);
-            acc.x += o.x;
-            acc.y |= o.y;
-        }
-    }
-    return acc;
-}
-
-__device__ __forceinline__ void warp_fill_actions(const uint8_t *__restrict__ actions, uint64_t seed, int env,
-                                                  int s0, int n_steps, uint8_t *acts, int &warn)
-{
-    const int lane = threadIdx.x & 31;
-    for (int k = lane; k < kActChunk; k += 32) {
-        const int s = s0 + k;
-        if (s < n_steps)
-            acts[s & (kActChunk - 1)] = (uint8_t)action_at(actions, seed, env, s, &warn);
-    }
-}
-
-// next = (D & ~CLEAR) | (~D & SET) in place over the tile planes; SET / CLEAR cleared.
-__device__ __forceinline__ void warp_combine(const DevConfig &cf, const WarpSmem &S)
-{
-    const int lane = threadIdx.x & 31;
-    for (int i = lane; i < cf.C * cf.NW; i += 32) {
-        const int c = i / cf.NW, w = i - c * cf.NW;
-        const uint32_t d = S.planes[c * cf.NWP + w].x, st = S.setp[i], cl = S.clrp[i];
-        S.setp[i] = 0u;
-        S.clrp[i] = 0u;
-        put_word(S.planes, cf.NWP, c, w, (d & ~cl) | (~d & st));
-    }
-}
-
 // Shared memory of expand_warp_kernel: one region per CTA (the rule table when
 // staged, valid-anchor masks, column masks), then per warp its planes, SET /
 // CLEAR / child planes and the canonical bytes of its five children.  All
@@ -860,6 +696,9 @@ struct ExpandLayout {
     size_t child_bytes;  // canonical bytes of one child, padded to 16
 };
 
+// Per warp: C tile planes and the force planes of the five actions (C + a),
+// doubled; SET and CLEAR planes per action; one child's planes; the five
+// children's canonical bytes.
 __host__ __device__ inline ExpandLayout expand_layout(const DevConfig &cf)
 {
     ExpandLayout L;
@@ -870,9 +709,9 @@ __host__ __device__ inline ExpandLayout expand_layout(const DevConfig &cf)
     L.warps = align16(L.rules + (size_t)cf.rule_words * 4);
     L.child_bytes = align16((size_t)cf.HW * cf.cell_bytes);
     L.planes = 0;
-    L.setp = align16((size_t)(cf.C + 1) * cf.NWP * 8);
-    L.clrp = align16(L.setp + pw);
-    L.basep = align16(L.clrp + pw);
+    L.setp = align16((size_t)(cf.C + 5) * cf.NWP * 8);
+    L.clrp = align16(L.setp + 5 * pw);
+    L.basep = align16(L.clrp + 5 * pw);
     L.bytes = align16(L.basep + pw);
     L.per_warp = align16(L.bytes + 5 * L.child_bytes);
     return L;
@@ -914,7 +753,109 @@ __device__ __forceinline__ int planes_to_cells(const DevConfig &cf, const uint32
     return __any_sync(0xffffffffu, goal) || cf.ch_goal < 0;
 }
 
-template <typename CellT, int NA, int RB, bool SM>
+// One parent's five children (one warp).  A parent's children differ only in
+// the force plane, so each rule's terms on tile channels are evaluated once
+// (pass 1, four terms per vote); a rule with anchors left then applies its
+// force terms for all five actions at once (pass 2) and writes each action's
+// outputs into that action's SET / CLEAR planes.
+template <typename CellT, int NA, bool SM>
+__device__ __forceinline__ void expand_rules(const DevConfig &cf, const uint32_t *tab, const WarpSmem &S,
+                                             int (&rew)[5])
+{
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const int NW = cf.NW;
+    const uint32_t plane_bytes = (uint32_t)cf.NWP * 8;
+    const uint32_t force0 = (uint32_t)cf.C * plane_bytes, force_end = force0 + plane_bytes;
+    const uint32_t pbase = (uint32_t)__cvta_generic_to_shared(S.planes) + q * 8;
+    const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+    const uint32_t cnw = (uint32_t)cf.C * NW;
+    for (int r = 0; r < cf.R; ++r) {
+        const uint4 h0 = ld4<SM>(tab + 4 + 8 * r);
+        const uint4 h1 = ld4<SM>(tab + 8 + 8 * r);
+        const uint32_t *vmr = S.vm + ((h1.z >> (8 * g)) & 0xffu) * NW;
+        uint32_t m[NA];
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            const int a = q + 8 * u;
+            m[u] = a < NW ? vmr[a] : 0u;
+        }
+        const uint2 *tp = terms + (size_t)h1.x * 4 + g;
+        const uint32_t nt = h0.x + h0.y;
+        // pass 1: tile-channel terms (a force term, or one past the end, passes)
+        bool live = __any_sync(0xffffffffu, (m[0] | (NA > 1 ? m[NA - 1] : 0u)) != 0u);
+        for (uint32_t t = 0; live && t < nt; t += 4) {
+            uint2 d[4];
+            bool skip[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                d[j] = t + j < nt ? ld2<SM>(tp + 4 * (t + j)) : make_uint2(force0, 0u);
+                skip[j] = d[j].x >= force0 && d[j].x < force_end;
+            }
+            uint32_t any = 0;
+#pragma unroll
+            for (int u = 0; u < NA; ++u) {
+                uint32_t x = m[u];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const uint2 w = lds2(pbase + (skip[j] ? 0u : d[j].x) + 64 * u);
+                    const uint32_t v = __funnelshift_r(w.x, w.y, d[j].y) ^ (uint32_t)((int32_t)d[j].y >> 31);
+                    x &= skip[j] ? 0xffffffffu : v;
+                }
+                m[u] = x;
+                any |= x;
+            }
+            live = __any_sync(0xffffffffu, any != 0u);
+        }
+        if (!live)
+            continue;
+        // pass 2: the force terms, for every action
+        uint32_t ma[5][NA];
+#pragma unroll
+        for (int a = 0; a < 5; ++a)
+#pragma unroll
+            for (int u = 0; u < NA; ++u)
+                ma[a][u] = m[u];
+        for (uint32_t t = 0; t < nt; ++t) {
+            const uint2 d = ld2<SM>(tp + 4 * t);
+            if (d.x < force0 || d.x >= force_end)  // the same for every rotation
+                continue;
+            const uint32_t neg = (uint32_t)((int32_t)d.y >> 31);
+#pragma unroll
+            for (int a = 0; a < 5; ++a)
+#pragma unroll
+                for (int u = 0; u < NA; ++u) {
+                    const uint2 w = lds2(pbase + d.x + (uint32_t)a * plane_bytes + 64 * u);
+                    ma[a][u] &= __funnelshift_r(w.x, w.y, d.y) ^ neg;
+                }
+        }
+        const uint4 *op = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, tab[1])) + (size_t)h1.y * 4 + g;
+#pragma unroll
+        for (int a = 0; a < 5; ++a) {
+            uint32_t cnt = 0;
+#pragma unroll
+            for (int u = 0; u < NA; ++u)
+                cnt += __popc(ma[a][u]);
+            if (cnt == 0)
+                continue;
+            rew[a] += (int)h0.w * (int)cnt;
+            for (uint32_t o = 0; o < h0.z; ++o) {
+                const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
+#pragma unroll
+                for (int u = 0; u < NA; ++u) {
+                    if (!ma[a][u])
+                        continue;
+                    const int w0 = q + 8 * u + (int)ov.x;
+                    const uint32_t lo = ma[a][u] << ov.y;
+                    const uint32_t hi = ov.y ? (ma[a][u] >> (32u - ov.y)) : 0u;
+                    scatter_bits(S.setp + a * cnw, ov.z, NW, w0, lo, hi);
+                    scatter_bits(S.clrp + a * cnw, ov.w, NW, w0, lo, hi);
+                }
+            }
+        }
+    }
+}
+
+template <typename CellT, int NA, bool SM>
 __global__ void __launch_bounds__(32 * kWarpCtaMax)
 expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
                    const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g,
@@ -965,9 +906,9 @@ expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint3
     S.cells = nullptr;
     uint32_t *bytes = reinterpret_cast<uint32_t *>(wr + L.bytes);
     const uint32_t *tab = SM ? rules : tab_g;
-    for (int i = lane; i < (C + 1) * NWP; i += 32)
+    for (int i = lane; i < (C + 5) * NWP; i += 32)
         S.planes[i] = make_uint2(0u, 0u);
-    for (int i = lane; i < C * NW; i += 32) {
+    for (int i = lane; i < 5 * C * NW; i += 32) {
         S.setp[i] = 0u;
         S.clrp[i] = 0u;
     }
@@ -976,29 +917,25 @@ expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint3
     if (mine) {
         warp_cells_to_planes<CellT>(cf, parents + (size_t)node * HW, S.planes, nullptr);
         __syncwarp();
+        force_planes(cf, S.planes, S.masks, 0, 1, C);
+        __syncwarp();
+        int rew[5] = {0, 0, 0, 0, 0};
+        expand_rules<CellT, NA, SM>(cf, tab, S, rew);
+        __syncwarp();  // every lane's SET / CLEAR bits
+#pragma unroll
         for (int a = 0; a < 5; ++a) {
-            force_plane(cf, S.planes, S.masks, a);
-            __syncwarp();
-            const int2 o = warp_rules<NA, RB, SM>(cf, tab, S);
-            const int rew = __reduce_add_sync(0xffffffffu, o.x);
-            __syncwarp();
-            const bool any = __any_sync(0xffffffffu, o.y != 0);
+            const uint32_t *st = S.setp + a * C * NW, *cl = S.clrp + a * C * NW;
             for (int i = lane; i < C * NW; i += 32) {  // child planes
                 const int c = i / NW, w = i - c * NW;
                 const uint32_t d = S.planes[c * NWP + w].x;
-                uint32_t v = d;
-                if (any) {
-                    v = (d & ~S.clrp[i]) | (~d & S.setp[i]);
-                    S.setp[i] = 0u;
-                    S.clrp[i] = 0u;
-                }
-                S.basep[i] = v;
+                S.basep[i] = (d & ~cl[i]) | (~d & st[i]);
             }
             __syncwarp();
             const int goal_left = planes_to_cells<CellT>(
                 cf, S.basep, bytes + a * (L.child_bytes / 4), children + ((size_t)node * 5 + a) * HW);
+            const int r = __reduce_add_sync(0xffffffffu, rew[a]);
             if (lane == 0) {
-                rewards[(size_t)node * 5 + a] = rew;
+                rewards[(size_t)node * 5 + a] = r;
                 if (done)
                     done[(size_t)node * 5 + a] = (uint8_t)!goal_left;
             }
@@ -1036,6 +973,13 @@ expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint3
         hashes[(size_t)nd * 5 + a] = hsh;
     }
 }
+
+// A lane's anchor words, passed by value (a register array would go to local
+// memory through a call).
+template <int NA>
+struct Words {
+    uint32_t v[NA];
+};
 
 // ============================================================ fast rollout
 // Boards of at most 16 plane words.  One CTA per environment with NWARP warps;
@@ -1084,41 +1028,6 @@ struct FastSmem {
     uint8_t *acts;
 };
 
-// Force planes of actions a0, a0 + stride, ... < 5 from the player plane (one
-// warp), into planes first + action.
-static __device__ void force_planes(const DevConfig &cf, uint2 *P, const uint32_t *masks, int a0, int stride,
-                                    int first)
-{
-    const int lane = threadIdx.x & 31, NW = cf.NW, NWP = cf.NWP;
-    const uint32_t *firstcol = masks, *lastcol = masks + NW, *cellmask = masks + 2 * NW;
-    const uint2 *pl = P + (cf.ch_player >= 0 ? cf.ch_player : 0) * NWP;
-    for (int action = a0; action < 5; action += stride)
-        for (int w = lane; w < NW; w += 32) {
-            uint32_t f = 0;
-            if (cf.ch_player >= 0 && action > 0) {
-                const int n = (action == 1 || action == 3) ? cf.W : 1;
-                const int q = n >> 5, r = n & 31;
-                if (action == 1 || action == 4) {
-                    const uint2 e = pl[w + q];
-                    f = __funnelshift_r(e.x, e.y, r);
-                } else {
-                    const int j = w - q;
-                    if (j >= 1) {
-                        const uint2 e = pl[j - 1];
-                        f = __funnelshift_l(e.x, e.y, r);
-                    } else if (j == 0) {
-                        f = pl[0].x << r;
-                    }
-                }
-                if (action == 2)
-                    f &= ~firstcol[w];
-                else if (action == 4)
-                    f &= ~lastcol[w];
-                f &= cellmask[w];
-            }
-            put_word(P, NWP, first + action, w, f);
-        }
-}
 
 // Terms t0.. of rule r, four per warp vote, then the rule's write.  `m` holds
 // the live anchors so far; force terms read `fdelta` bytes past the action-0
@@ -1190,12 +1099,6 @@ __device__ __noinline__ int2 fast_rule_rest(const DevConfig &cf, const uint32_t 
     return make_int2((int)h0.w * (int)cnt, 1);
 }
 
-__device__ __forceinline__ uint2 lds2(uint32_t addr)
-{
-    uint2 v;
-    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
-    return v;
-}
 
 // Per-lane register data of one owned rule.
 template <int NA>
