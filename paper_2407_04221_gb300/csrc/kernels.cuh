@@ -697,8 +697,8 @@ struct ExpandLayout {
 };
 
 // Per warp: C tile planes and the force planes of the five actions (C + a),
-// doubled; SET and CLEAR planes per action; one child's planes; the five
-// children's canonical bytes.
+// doubled; SET and CLEAR planes per action; the five children's canonical
+// bytes.
 __host__ __device__ inline ExpandLayout expand_layout(const DevConfig &cf)
 {
     ExpandLayout L;
@@ -711,22 +711,23 @@ __host__ __device__ inline ExpandLayout expand_layout(const DevConfig &cf)
     L.planes = 0;
     L.setp = align16((size_t)(cf.C + 5) * cf.NWP * 8);
     L.clrp = align16(L.setp + 5 * pw);
-    L.basep = align16(L.clrp + 5 * pw);
-    L.bytes = align16(L.basep + pw);
+    L.basep = L.clrp;  // not used
+    L.bytes = align16(L.clrp + 5 * pw);
     L.per_warp = align16(L.bytes + 5 * L.child_bytes);
     return L;
 }
 
-// Cells of a board from its flat planes (C words per plane word), written as
-// canonical bytes to `out` (shared, 16-byte aligned) and to `dst` (global),
+// Cells of a child board, (D & ~CLEAR) | (~D & SET) from the parent's doubled
+// planes and the child's SET / CLEAR planes, written as canonical bytes to
+// `out` (shared, 16-byte aligned) and to `dst` (global),
 // and whether any goal tile is left.  One warp; a 32-bit word per lane per
 // pass: four 1-byte cells (bit k of a channel's 4-bit slice spread to byte k
 // by a multiply) or two 2-byte cells.
 template <typename CellT>
-__device__ __forceinline__ int planes_to_cells(const DevConfig &cf, const uint32_t *flat, uint32_t *out,
-                                               CellT *dst)
+__device__ __forceinline__ int planes_to_cells(const DevConfig &cf, const uint2 *dbl, const uint32_t *setp,
+                                               const uint32_t *clrp, uint32_t *out, CellT *dst)
 {
-    const int lane = threadIdx.x & 31, HW = cf.HW, NW = cf.NW;
+    const int lane = threadIdx.x & 31, HW = cf.HW, NW = cf.NW, NWP = cf.NWP;
     constexpr int kPer = 4 / (int)sizeof(CellT);  // cells per 32-bit word
     const int n_words = (HW + kPer - 1) / kPer;
     const bool aligned = (HW % kPer) == 0 && (reinterpret_cast<uintptr_t>(dst) & 3u) == 0;
@@ -735,7 +736,8 @@ __device__ __forceinline__ int planes_to_cells(const DevConfig &cf, const uint32
         const int p0 = g * kPer, j = p0 >> 5, b = p0 & 31;
         uint32_t v = 0;
         for (int c = 0; c < cf.C; ++c) {
-            const uint32_t x = flat[c * NW + j] >> b;
+            const uint32_t d = dbl[c * NWP + j].x, st = setp[c * NW + j], cl = clrp[c * NW + j];
+            const uint32_t x = ((d & ~cl) | (~d & st)) >> b;  // the child's word
             const uint32_t spread = sizeof(CellT) == 1 ? ((x & 0xfu) * 0x00204081u) & 0x01010101u
                                                        : ((x & 0x3u) * 0x00008001u) & 0x00010001u;
             v |= spread << c;
@@ -924,15 +926,9 @@ expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint3
         __syncwarp();  // every lane's SET / CLEAR bits
 #pragma unroll
         for (int a = 0; a < 5; ++a) {
-            const uint32_t *st = S.setp + a * C * NW, *cl = S.clrp + a * C * NW;
-            for (int i = lane; i < C * NW; i += 32) {  // child planes
-                const int c = i / NW, w = i - c * NW;
-                const uint32_t d = S.planes[c * NWP + w].x;
-                S.basep[i] = (d & ~cl[i]) | (~d & st[i]);
-            }
-            __syncwarp();
-            const int goal_left = planes_to_cells<CellT>(
-                cf, S.basep, bytes + a * (L.child_bytes / 4), children + ((size_t)node * 5 + a) * HW);
+            const int goal_left = planes_to_cells<CellT>(cf, S.planes, S.setp + a * C * NW, S.clrp + a * C * NW,
+                                                         bytes + a * (L.child_bytes / 4),
+                                                         children + ((size_t)node * 5 + a) * HW);
             const int r = __reduce_add_sync(0xffffffffu, rew[a]);
             if (lane == 0) {
                 rewards[(size_t)node * 5 + a] = r;
