@@ -53,12 +53,12 @@ void launch_select_hash(const DevConfig &cf, int cap, uint32_t vmask, int F, con
 {
     const size_t sm = select_hash_smem_bytes(F);
     if (cf.cell_bytes == 1)
-        select_hash_kernel<uint8_t><<<cf.B, kThreads, sm, st>>>(
+        select_hash_kernel<uint8_t><<<cf.B, kSelectThreads, sm, st>>>(
             cf, cap, vmask, F, n_parent, parent_cum, parent_live, (const uint8_t *)cand_grids, cand_reward,
             cand_done, cand_hash, k, (uint8_t *)next_grids, next_cum, next_hash, next_live, n_next, vtab, vzero,
             n_visited, status);
     else
-        select_hash_kernel<uint16_t><<<cf.B, kThreads, sm, st>>>(
+        select_hash_kernel<uint16_t><<<cf.B, kSelectThreads, sm, st>>>(
             cf, cap, vmask, F, n_parent, parent_cum, parent_live, (const uint16_t *)cand_grids, cand_reward,
             cand_done, cand_hash, k, (uint16_t *)next_grids, next_cum, next_hash, next_live, n_next, vtab, vzero,
             n_visited, status);

@@ -2171,8 +2171,10 @@ inline size_t select_hash_smem_bytes(int F)
     return (size_t)select_hash_slots(F) * 16 + (size_t)n2 * sizeof(Key128) + 64;
 }
 
+constexpr int kSelectThreads = 1024;  // threads of select_hash_kernel (one CTA per env)
+
 template <typename CellT>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kSelectThreads)
 select_hash_kernel(DevConfig cf, int cap, uint32_t vmask, int F, const int32_t *__restrict__ n_parent,
                    const int32_t *__restrict__ parent_cum, const uint8_t *__restrict__ parent_live,
                    const CellT *__restrict__ cand_grids, const int32_t *__restrict__ cand_reward,
