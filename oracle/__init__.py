@@ -64,6 +64,10 @@ def lib():
         L.or_expand.argtypes = [vp, vp, i32, vp, vp, i32, vp, vp, vp, vp, i32]
         L.or_search.restype = i32
         L.or_search.argtypes = [vp, vp, i32, vp, vp, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, i32]
+        L.or_observe.restype = i32
+        L.or_observe.argtypes = [vp, i32, vp, i32, vp, vp]
+        L.or_rule_obs.restype = i32
+        L.or_rule_obs.argtypes = [vp, vp, i32, vp, vp]
         _lib = L
     return _lib
 
@@ -211,3 +215,27 @@ def search(cfg: OrCfg, rules, roots, iterations, k, env_ids=None, threads=None):
     assert rc == 0, rc
     return dict(grids=fg, cum=fc, hash=fh, done=fd, n=nf, trace_n=tn[:, :iterations],
                 trace_best=tb[:, :iterations], n_visited=nv)
+
+
+def observe(cfg: OrCfg, grids, window: int):
+    """Player-centred patches of boards [n, H, W] -> (obs [n, window, window, C] uint8,
+    player_yx [n, 2] int32, (-1, -1) where no player is on the board)."""
+    grids = np.ascontiguousarray(grids, dtype=cell_dtype(cfg.C))
+    n = grids.shape[0]
+    obs = np.zeros((n, window, window, cfg.C), np.uint8)
+    pyx = np.zeros((n, 2), np.int32)
+    rc = lib().or_observe(ctypes.byref(cfg), n, _p(grids), int(window), _p(obs), _p(pyx))
+    assert rc == 0, rc
+    return obs, pyx
+
+
+def rule_obs(cfg: OrCfg, rules):
+    """Binary form of rule tables [T, R] records -> (bits [T, R, 4, 5, 5, C+1] uint8,
+    reward [T, R] int32)."""
+    rb = _rules_buf(rules)
+    T = rb.size // (408 * max(cfg.n_rules, 1)) if cfg.n_rules else 0
+    bits = np.zeros((T, cfg.n_rules, 4, 5, 5, cfg.C + 1), np.uint8)
+    rew = np.zeros((T, cfg.n_rules), np.int32)
+    rc = lib().or_rule_obs(ctypes.byref(cfg), _p(rb), T, _p(bits), _p(rew))
+    assert rc == 0, rc
+    return bits, rew

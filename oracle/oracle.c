@@ -805,3 +805,89 @@ int or_search(const or_cfg *cfg, const uint8_t *rules, int n, const int32_t *env
                     trace_best, n_visited};
     return run_pool(n, threads, &j, search_item);
 }
+
+/* ------------------------------------------------- policy observation
+ * Sec. 3.2 (imitation learning): the agent observes a local patch of tiles
+ * centred on the player's current position, together with a binary form of
+ * the environment's rules.  Sec. 4, Table 1, varies the patch width (5, 10,
+ * 20, 31) and pads the map with zeros where the patch leaves it; Table 2
+ * hides the rules by putting zeros in their place.
+ *
+ * Readings (the paper says no more):
+ *  - the player is the first cell in row-major order that holds the player
+ *    bit; with no such cell every entry of the patch is 0;
+ *  - patch entry (i, k) is board cell (py - window/2 + i, px - window/2 + k),
+ *    integer division, so the player sits at (window/2, window/2) and a
+ *    patch 2*max(H, W) - 1 wide holds the whole board wherever the player is;
+ *  - cells outside the board read as 0 in every channel;
+ *  - the patch is written channels-last as bytes [window][window][C]: byte c
+ *    of an entry is tile bit c (force is never stored, so never observed).
+ * player_yx (nullable) receives (py, px), or (-1, -1) without a player. */
+int or_observe(const or_cfg *cfg, int n, const void *grids, int window, uint8_t *obs,
+               int32_t *player_yx)
+{
+    if (check_cfg(cfg) || n < 0 || window < 1 || cfg->ch_player < 0 || cfg->ch_player >= cfg->C)
+        return -1;
+    const int H = cfg->H, W = cfg->W, C = cfg->C;
+    uint32_t cells[OR_MAXCELLS];
+    for (int b = 0; b < n; b++) {
+        load_grid((const uint8_t *)grids + (size_t)b * grid_bytes(cfg), H, W, C, cells);
+        int py = -1, px = -1;
+        for (int q = 0; q < H * W && py < 0; q++)
+            if ((cells[q] >> cfg->ch_player) & 1u) {
+                py = q / W;
+                px = q % W;
+            }
+        uint8_t *o = obs + (size_t)b * window * window * C;
+        for (int i = 0; i < window; i++)
+            for (int k = 0; k < window; k++) {
+                int y = py - window / 2 + i, x = px - window / 2 + k;
+                int on_board = py >= 0 && y >= 0 && y < H && x >= 0 && x < W;
+                for (int c = 0; c < C; c++)
+                    o[((size_t)i * window + k) * C + c] =
+                        on_board ? (uint8_t)((cells[y * W + x] >> c) & 1u) : 0;
+            }
+        if (player_yx) {
+            player_yx[2 * b] = py;
+            player_yx[2 * b + 1] = px;
+        }
+    }
+    return 0;
+}
+
+/* Binary form of the rules (Sec. 3.2).  Reading: every rule becomes four
+ * binary planes over a 5 x 5 frame with C + 1 channels (force last):
+ * plane 0 the present entries and plane 1 the absent entries of the input
+ * pattern (the +1 and -1 weights of the matching kernel, Sec. 2.1), plane 2
+ * the set entries and plane 3 the clear entries of the output pattern (tile
+ * channels only, so their force channel is 0).  Entry (i, k) of the base,
+ * unrotated h x w pattern sits at frame row i, column k; the rest of the
+ * frame is 0.  bits: [n_tables][R][4][5][5][C+1]; reward (nullable):
+ * [n_tables][R], the rule's reward as given. */
+int or_rule_obs(const or_cfg *cfg, const uint8_t *rules, int n_tables, uint8_t *bits,
+                int32_t *reward)
+{
+    if (check_cfg(cfg) || n_tables < 0)
+        return -1;
+    const int R = cfg->n_rules, NCH = cfg->C + 1;
+    for (int t = 0; t < n_tables; t++)
+        for (int r = 0; r < R; r++) {
+            or_pattern p;
+            parse_rule(rules + ((size_t)t * R + r) * OR_RULE_BYTES, &p);
+            uint8_t *o = bits + ((size_t)t * R + r) * 4 * 25 * NCH;
+            memset(o, 0, (size_t)4 * 25 * NCH);
+            for (int i = 0; i < p.h; i++)
+                for (int k = 0; k < p.w; k++) {
+                    const int e = i * p.w + k, f = i * 5 + k;
+                    for (int c = 0; c < NCH; c++) {
+                        o[(0 * 25 + f) * NCH + c] = (p.present[e] >> c) & 1u;
+                        o[(1 * 25 + f) * NCH + c] = (p.absent[e] >> c) & 1u;
+                        o[(2 * 25 + f) * NCH + c] = c < cfg->C ? (p.set[e] >> c) & 1u : 0;
+                        o[(3 * 25 + f) * NCH + c] = c < cfg->C ? (p.clear[e] >> c) & 1u : 0;
+                    }
+                }
+            if (reward)
+                reward[(size_t)t * R + r] = p.reward;
+        }
+    return 0;
+}
