@@ -199,9 +199,9 @@ def profile_path(kernel: str, wl) -> str:
     return os.path.join(PROFILE_DIR, f"{kernel}_{wl.name}.md")
 
 
-def profile_traffic(kernel: str, wl) -> float | None:
+def profile_traffic(kernel: str, wl, src: str = KERNEL_SRC) -> float | None:
     """DRAM bytes per launch from the committed ncu summary of this kernel on
-    this workload, if it was taken on the current kernel source."""
+    this workload, if it was taken on the current kernel source `src`."""
     try:
         text = open(profile_path(kernel, wl)).read()
     except OSError:
@@ -210,7 +210,7 @@ def profile_traffic(kernel: str, wl) -> float | None:
     t = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
     if not m or not t:
         return None
-    cur = hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()
+    cur = hashlib.sha256(open(src, "rb").read()).hexdigest()
     return float(t.group(1)) if cur.startswith(m.group(1)) else None
 
 
@@ -657,6 +657,215 @@ def run_search_reference(args, wl):
     return 0
 
 
+# ------------------------------------------------- policy observation
+OBSERVE_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_observe.cu")
+OBSERVE_ROLLOUT_STEPS = 60  # boards observed after this many random steps (multi-hot cells)
+
+
+class ObserveWorkload:
+    """Player-centred patches (av_observe) of the 16,384 boards of the
+    training shape (16 x 16, C = 10) for one window width."""
+
+    def __init__(self, base: wk.Workload, window: int):
+        self.base, self.window = base, window
+        self.name = f"observe-w{window}-grid{base.H}-b{base.batch}-c{base.C}"
+
+    def bytes_per_obs(self) -> int:
+        b = self.base
+        return b.H * b.W * b.cell_bytes + self.window * self.window * b.C
+
+    def config(self, sample=None) -> dict:
+        b = self.base
+        d = {"workload": self.name, "batch": b.batch, "H": b.H, "W": b.W, "tile_channels": b.C,
+             "window": self.window, "obs_layout": "uint8 [B][window][window][C], channels last",
+             "boards": f"reset, then {OBSERVE_ROLLOUT_STEPS} random-action steps of the"
+                       f" {b.n_rules}-rule tables",
+             "l2": "flushed (256 MiB write) between timed launches", "parallelism": "replicas"}
+        if sample:
+            d["sample_envs"] = sample
+        return d
+
+
+def observe_boards(wl: ObserveWorkload, seed: int, env=None):
+    """(env, boards after the warm-up rollout) for the observation benchmark."""
+    s = wk.seeds(seed)
+    env.reset(s["reset"])
+    env.rollout(OBSERVE_ROLLOUT_STEPS, s["actions"])
+    g, _ = env.get_state()
+    return g
+
+
+def observe_cpu_baseline(cfg, boards_np, window, budget_s: float = 4.0) -> dict:
+    """The oracle's observation (one thread), repeated over the whole batch."""
+    import oracle
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        oracle.observe(cfg, boards_np, window)
+        reps += 1
+        dt = time.perf_counter() - t0
+        if dt > budget_s:
+            break
+    n = boards_np.shape[0]
+    return {"value": reps * n / dt, "unit": "observations/s", "cores": 1, "kind": "oracle",
+            "sample": f"all {n} boards x {reps} passes", "seconds": dt}
+
+
+def run_observe(args, wl: ObserveWorkload):
+    """One benchmark step = one av_observe launch over every board."""
+    import torch
+
+    import paper_2407_04221_gb300 as av
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    seed = args.seed + 1000 * rank
+    base = wl.base
+    _, rules, cum = wk.make(base, seed)
+    fields = wk.config_fields(base)
+    env = av.Env(fields, rules, cum, device=dev)
+    boards = observe_boards(wl, seed, env)
+    B, w = base.batch, wl.window
+    obs = torch.empty(B, w, w, base.C, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        av.av_observe(env.h, None, w, obs, None, stream)
+    torch.cuda.synchronize(dev)
+    env.sync()
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(torch.cuda.current_device() if world == 1 else local)
+    sampler.start()
+    barrier()
+    sampler.mark_start()
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.fill_(i & 0xff)
+        starts[i].record(stream)
+        av.av_observe(env.h, None, w, obs, None, stream)
+        ends[i].record(stream)
+    barrier()
+    wall = time.perf_counter() - t_wall
+    sampler.mark_end()
+    clocks = sampler.stop()
+    env.sync()
+    ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
+    kernel_ms = sum(ms) / len(ms)
+    total_ms = max_over_ranks(sum(ms), world, dev)
+    value = B * args.steps * world / (total_ms / 1e3)
+
+    # ---- e2e: boards from pinned host memory in, observations to pinned host memory out
+    host_in = boards.cpu().pin_memory()
+    host_out = torch.empty(obs.shape, dtype=torch.uint8).pin_memory()
+    dev_in = torch.empty_like(boards)
+    e2e_steps = max(3, min(args.steps, 10))
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        dev_in.copy_(host_in, non_blocking=True)
+        av.av_observe(env.h, dev_in, w, obs, None, stream)
+        host_out.copy_(obs, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
+    e2e_value = B * world / (e2e_ms / 1e3)
+
+    if rank == 0:
+        peaks = measured_peaks()
+        peak = float(peaks.get("hbm_gbs", 6800.0))
+        per_obs = wl.bytes_per_obs()
+        achieved = per_obs * B / (kernel_ms / 1e3) / 1e9
+        line = {
+            "metric": "observations/s", "value": value, "unit": "observations/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u8", "data": "synthetic", "config": wl.config(),
+            "e2e": {"value": e2e_value, "unit": "observations/s",
+                    "h2d_bytes_per_step": int(host_in.numel() * host_in.element_size()),
+                    "d2h_bytes_per_step": int(host_out.numel())},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak,
+                         "traffic": profile_traffic("observe_kernel", wl, OBSERVE_SRC),
+                         "kernel": "observe_kernel", "bytes_per_obs": per_obs,
+                         "bytes_basis": "board read once (H*W cell bytes) + patch written once"
+                                        " (window^2 * C bytes)",
+                         "peak_from": "hbm_gbs of measured peaks" if "hbm_gbs" in peaks
+                                      else "fallback 6800 GB/s"},
+            "gpu_launches": args.steps,
+            "wall_s_timed_region": wall,
+        }
+        if clocks:
+            line["clocks"] = clocks
+        if world == 1 and not args.no_cpu_baseline:
+            import oracle
+            line["cpu_baseline"] = observe_cpu_baseline(oracle.make_cfg(**fields),
+                                                        gpu_boards_np(boards), w)
+        print(json.dumps(line))
+    env.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def gpu_boards_np(t) -> np.ndarray:
+    a = t.cpu().numpy()
+    return a.view(np.uint16) if a.dtype == np.int16 else a
+
+
+def run_observe_reference(args, wl: ObserveWorkload):
+    """The oracle's observation on the host, on the same boards (made by the
+    oracle's own rollout of the same seeds), one thread."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    base = wl.base
+    _, rules, cum = wk.make(base, args.seed)
+    cfg = oracle.make_cfg(**wk.config_fields(base))
+    s = wk.seeds(args.seed)
+    n = min(base.batch, 2048)
+    ids = np.arange(n)
+    g = oracle.reset(cfg, cum, s["reset"], ids)
+    g = oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), OBSERVE_ROLLOUT_STEPS,
+                       s["actions"], env_ids=ids)["grids"]
+    for _ in range(args.warmup):
+        oracle.observe(cfg, g[:64], wl.window)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.observe(cfg, g, wl.window)
+        times.append(time.perf_counter() - t0)
+    mean = sum(times) / len(times)
+    value = n / mean
+    line = {
+        "impl": "reference", "metric": "observations/s", "value": value,
+        "unit": "observations/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": mean * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u8", "data": "synthetic", "config": wl.config(sample=n),
+        "cpu_baseline": {"value": value, "unit": "observations/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{n} of {base.batch} boards per step"},
+        "e2e": {"value": value, "unit": "observations/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
 def run_int_probe() -> int:
     """Build and run the integer-issue probe (needs nvcc and a GPU)."""
     import tempfile
@@ -682,11 +891,20 @@ def main(argv=None):
     ap.add_argument("--fused-steps", type=int, default=0,
                     help="run a smaller case of the workload (profiling): steps per launch")
     ap.add_argument("--int-probe", action="store_true", help="measure integer issue rate and exit")
+    ap.add_argument("--observe", type=int, default=0, metavar="WINDOW",
+                    help="time av_observe (player-centred patches of this width) on the"
+                         " 16,384-env training shape instead of a rollout")
     args = ap.parse_args(argv)
     if args.int_probe:
         return run_int_probe()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.observe:
+        base = workload_for(3)
+        if args.batch > 0:
+            base = base.scaled(batch=args.batch)
+        owl = ObserveWorkload(base, args.observe)
+        return run_observe_reference(args, owl) if args.impl == "reference" else run_observe(args, owl)
     wl = workload_for(args.config)
     if args.batch > 0:
         wl = wl.scaled(batch=args.batch)

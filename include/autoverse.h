@@ -66,6 +66,7 @@ enum { AV_WARN_ACTION = 1 /* an action value >= 5 was treated as no-op */ };
 #define AV_MAX_C 16      /* C <= 16 tile channels (+1 force channel)     */
 #define AV_MAX_PATTERN 5 /* rule patterns up to 5 x 5                    */
 #define AV_MAX_RULES 64  /* rules per table                              */
+#define AV_MAX_WINDOW 127 /* observation patches up to 127 x 127 (2 * AV_MAX_SIDE - 1) */
 
 typedef struct av_handle av_handle; /* opaque; owns all env state on the device */
 
@@ -156,6 +157,34 @@ int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_tr
 int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_parent,
               void *children, int32_t *rewards, uint8_t *done, uint64_t *hashes,
               uintptr_t stream);
+
+/* Policy observation of each board (Sec. 3.2, imitation learning: the agent
+ * observes a local patch of tiles centred on the player's position; Sec. 4,
+ * Table 1: patch widths 5, 10, 20 and 31, the map padded with zeros where the
+ * patch leaves it).  grids: device [B][H][W] boards, or NULL for the handle's
+ * current boards.  obs: device uint8 [B][window][window][C], channels last:
+ * byte c of patch entry (i, k) is tile bit c of board cell
+ * (py - window/2 + i, px - window/2 + k) (integer division), 0 outside the
+ * board; (py, px) is the first row-major cell holding the player bit, and a
+ * board without one gives an all-zero patch.  A window of 2 * max(H, W) - 1
+ * holds the whole board wherever the player stands.  player_yx: device
+ * int32 [B][2] or NULL, receives (py, px), or (-1, -1) without a player.
+ * Any alignment of obs is accepted.  AV_EINVAL for window outside
+ * 1..AV_MAX_WINDOW or a NULL obs; AV_ESTATE when cfg.ch_player is -1. */
+int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, int32_t *player_yx,
+               uintptr_t stream);
+
+/* Binary form of the handle's rule tables (Sec. 3.2: the observation holds a
+ * binary representation of the environment's rules; Sec. 4, Table 2 hides
+ * them by zeros).  bits: device uint8 [T][R][4][5][5][C+1], T = B when
+ * rules_per_env else 1: plane 0 the present and plane 1 the absent entries of
+ * the input pattern, plane 2 the set and plane 3 the clear entries of the
+ * output pattern; entry (i, k) of the unrotated h x w pattern at frame row i,
+ * column k, byte c = channel c (C = force, always 0 in planes 2 and 3), 0
+ * outside the pattern.  reward: device int32 [T][R] or NULL, the rules'
+ * rewards.  The tables do not change, so one call per handle suffices.
+ * AV_EINVAL for a NULL bits with R > 0. */
+int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream);
 
 /* Start a search from the root boards roots (device [B][H][W]): writes
  * root_hash uint64[B] (FNV-1a 64 as in av_expand) and root_live uint8[B]

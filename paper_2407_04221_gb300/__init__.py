@@ -24,7 +24,9 @@ AV_PATH_BLOCK, AV_PATH_FAST, AV_PATH_WARP = 1, 2, 3
 RULE_BYTES = 408
 EXPORTS = ("av_create", "av_destroy", "av_reset", "av_set_state", "av_get_state", "av_step",
            "av_rollout", "av_expand", "av_search_init", "av_select", "av_select_static", "av_sync",
-           "av_warnings", "av_rollout_path", "av_strerror", "av_last_error")
+           "av_warnings", "av_rollout_path", "av_observe", "av_rule_obs", "av_strerror",
+           "av_last_error")
+AV_MAX_WINDOW = 127
 AV_SELECT_STATIC_MAX_HASHES = 1 << 21
 
 
@@ -74,6 +76,8 @@ def load() -> ctypes.CDLL:
         "av_sync": [vp],
         "av_warnings": [vp, ctypes.POINTER(ctypes.c_uint32)],
         "av_rollout_path": [vp, ctypes.POINTER(ctypes.c_int32)],
+        "av_observe": [vp, vp, i32, vp, vp, up],
+        "av_rule_obs": [vp, vp, vp, up],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -225,6 +229,18 @@ def av_rollout_path(h) -> int:
     return int(path.value)
 
 
+def av_observe(h, grids, window: int, obs, player_yx=None, stream=None):
+    """Player-centred patches (Sec. 3.2): obs [B, window, window, C] uint8;
+    grids None observes the handle's current boards."""
+    _check(h, "av_observe", load().av_observe(h, _ptr(grids), int(window), _ptr(obs),
+                                              _ptr(player_yx), _stream(stream)))
+
+
+def av_rule_obs(h, bits, reward=None, stream=None):
+    """Binary form of the rule tables: bits [T, R, 4, 5, 5, C+1] uint8, reward [T, R]."""
+    _check(h, "av_rule_obs", load().av_rule_obs(h, _ptr(bits), _ptr(reward), _stream(stream)))
+
+
 class Env:
     """Owns one handle; allocates output tensors on demand (torch, cuda)."""
 
@@ -339,6 +355,26 @@ class Env:
             trace_best[:, it].copy_(cum[:, 0])
         return dict(grids=front, cum=cum, hash=hsh, live=live, n=n, trace_n=trace_n,
                     trace_best=trace_best)
+
+    def observe(self, window: int, grids=None, stream=None):
+        """Player-centred patches of the current boards (or of `grids`
+        [B, H, W]) -> (obs [B, window, window, C] uint8, player_yx [B, 2])."""
+        import torch
+        obs = torch.empty(self.B, window, window, self.C, dtype=torch.uint8, device=self.device)
+        pyx = torch.empty(self.B, 2, dtype=torch.int32, device=self.device)
+        av_observe(self.h, grids, window, obs, pyx, stream)
+        return obs, pyx
+
+    def rule_obs(self, stream=None):
+        """-> (bits [T, R, 4, 5, 5, C+1] uint8, reward [T, R] int32), T = B
+        with per-env rules, else 1."""
+        import torch
+        T = self.B if int(self.cfg["rules_per_env"]) else 1
+        R = int(self.cfg["n_rules"])
+        bits = torch.empty(T, R, 4, 5, 5, self.C + 1, dtype=torch.uint8, device=self.device)
+        rew = torch.empty(T, R, dtype=torch.int32, device=self.device)
+        av_rule_obs(self.h, bits, rew, stream)
+        return bits, rew
 
     def sync(self):
         av_sync(self.h)

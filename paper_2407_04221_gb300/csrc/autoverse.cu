@@ -43,6 +43,7 @@ struct av_handle {
     uint32_t *d_vzero = nullptr;    // [B] 1 if the state whose hash is 0 was visited
     int32_t *d_n_visited = nullptr; // [B]
     uint32_t vis_mask = 0;          // slots per env - 1 (a power of two >= 2 x capacity, minus one)
+    uint32_t *d_rules = nullptr;    // the packed 408-byte records as given, [n_tables][R] (rule observation)
     bool has_cum = false;
     std::string last_error;
 };
@@ -372,6 +373,7 @@ void free_all(av_handle *h)
     cudaFree(h->d_vtab);
     cudaFree(h->d_vzero);
     cudaFree(h->d_n_visited);
+    cudaFree(h->d_rules);
 }
 
 cudaStream_t as_stream(uintptr_t s) { return reinterpret_cast<cudaStream_t>(s); }
@@ -504,7 +506,8 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
         (rc = dalloc(h, &h->d_vm, vm.size())) || (rc = dalloc(h, &h->d_masks, masks.size())) ||
         (rc = dalloc(h, (uint8_t **)&h->d_cur, B * h->grid_bytes)) ||
         (rc = dalloc(h, (uint8_t **)&h->d_init, B * h->grid_bytes)) || (rc = dalloc(h, &h->d_t, B)) ||
-        (rc = dalloc(h, &h->d_status, 4))) {
+        (rc = dalloc(h, &h->d_status, 4)) ||
+        (rc = dalloc(h, (uint8_t **)&h->d_rules, (size_t)n_tables * cfg->n_rules * sizeof(av_rule)))) {
         free_all(h);
         delete h;
         return rc;
@@ -537,6 +540,8 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     if (e == cudaSuccess) e = cudaMemcpy(h->d_tab_off, tab_off.data(), tab_off.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(h->d_vm, vm.data(), vm.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(h->d_masks, masks.data(), masks.size() * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && cfg->n_rules > 0)
+        e = cudaMemcpy(h->d_rules, rules, (size_t)n_tables * cfg->n_rules * sizeof(av_rule), cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemset(h->d_cur, 0, B * h->grid_bytes);
     if (e == cudaSuccess) e = cudaMemset(h->d_init, 0, B * h->grid_bytes);
     if (e == cudaSuccess) e = cudaMemset(h->d_t, 0, B * 4);
@@ -640,6 +645,32 @@ int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_par
     launch_expand(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, parents, F, n_parent, children, rewards,
                   done, hashes, as_stream(stream));
     return launch_check(h, "expand kernel");
+}
+
+int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, int32_t *player_yx,
+               uintptr_t stream)
+{
+    if (!h || !obs)
+        return AV_EINVAL;
+    if (window < 1 || window > AV_MAX_WINDOW)
+        return fail(h, AV_EINVAL, "av_observe: window must be in 1..AV_MAX_WINDOW");
+    if (h->cf.ch_player < 0)
+        return fail(h, AV_ESTATE, "av_observe: the configuration has no player channel");
+    if ((size_t)h->cf.B > 0x7fffffffu)
+        return AV_EINVAL;
+    launch_observe(h->cf, grids ? grids : h->d_cur, window, obs, player_yx, as_stream(stream));
+    return launch_check(h, "observe kernel");
+}
+
+int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream)
+{
+    if (!h || (!bits && h->cf.R > 0))
+        return AV_EINVAL;
+    const size_t n = (size_t)h->n_tables * h->cf.R;
+    if (n * 100 > 0x7fffffffu)
+        return AV_EINVAL;
+    launch_rule_obs((int)n, h->cf.C, h->d_rules, bits, reward, as_stream(stream));
+    return launch_check(h, "rule observation kernel");
 }
 
 int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t *root_live,

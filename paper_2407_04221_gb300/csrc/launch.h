@@ -18,6 +18,7 @@ cudaError_t configure_warp_u16();
 cudaError_t configure_block();
 cudaError_t configure_expand();
 cudaError_t configure_search();
+cudaError_t configure_observe();
 
 void launch_rollout_fast_u8(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
                             const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
@@ -64,6 +65,14 @@ void launch_select(const DevConfig &cf, int cap, int parity, int F, const int32_
                    void *next_grids, int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live,
                    int32_t *n_next, uint64_t *visited, int32_t *n_visited, uint32_t *status, cudaStream_t st);
 
+// Policy observation (k_observe.cu).
+int observe_rows_per_slab(int window, int C);
+size_t observe_smem_bytes(const DevConfig &cf, int window);
+void launch_observe(const DevConfig &cf, const void *grids, int window, uint8_t *obs, int32_t *player_yx,
+                    cudaStream_t st);
+void launch_rule_obs(int n_rules_total, int C, const uint32_t *rules, uint8_t *bits, int32_t *reward,
+                     cudaStream_t st);
+
 inline cudaError_t configure_kernels()
 {
     cudaError_t e = configure_fast_u8();
@@ -73,6 +82,7 @@ inline cudaError_t configure_kernels()
     if (e == cudaSuccess) e = configure_block();
     if (e == cudaSuccess) e = configure_expand();
     if (e == cudaSuccess) e = configure_search();
+    if (e == cudaSuccess) e = configure_observe();
     return e;
 }
 
