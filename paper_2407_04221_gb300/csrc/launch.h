@@ -67,7 +67,6 @@ void launch_select(const DevConfig &cf, int cap, int parity, int F, const int32_
 
 // Policy observation (k_observe.cu).
 int observe_rows_per_slab(int window, int C);
-size_t observe_smem_bytes(const DevConfig &cf, int window);
 void launch_observe(const DevConfig &cf, const void *grids, int window, uint8_t *obs, int32_t *player_yx,
                     cudaStream_t st);
 void launch_rule_obs(int n_rules_total, int C, const uint32_t *rules, uint8_t *bits, int32_t *reward,

@@ -74,6 +74,28 @@ def test_random_boards_every_window(H, W, C):
     env.close()
 
 
+@pytest.mark.parametrize("B,H,W,C,window", [
+    (5000, 7, 9, 5, 3),       # 63-byte boards: plain loads; ~2 envs per CTA
+    (6000, 16, 16, 8, 31),    # 256-byte boards: asynchronous 16-byte copies
+    (700, 33, 33, 12, 127),   # seven row slabs per patch, several patches per CTA
+])
+def test_many_envs_per_cta(B, H, W, C, window):
+    """More environments than resident CTAs: each CTA runs several patches
+    through its two board buffers and two staging slabs."""
+    import paper_2407_04221_gb300 as av
+    rng = np.random.default_rng(B + window)
+    boards = _random_boards(rng, B, H, W, C, 0)
+    fields = _fields(B, H, W, C, 0)
+    env = av.Env(fields, np.zeros(0, np.uint8))
+    env.set_state(to_dev(boards))
+    obs, pyx = env.observe(window)
+    want, want_pyx = oracle.observe(oracle.make_cfg(**fields), boards, window)
+    np.testing.assert_array_equal(to_np(obs), want)
+    np.testing.assert_array_equal(to_np(pyx), want_pyx)
+    env.sync()
+    env.close()
+
+
 @pytest.mark.parametrize("offset", list(range(16)))
 def test_any_output_alignment_and_no_stray_writes(offset):
     """Patches written at every byte offset from a 16-byte boundary; the bytes
