@@ -24,6 +24,13 @@ FIELDS = ("batch", "H", "W", "C", "n_rules", "rules_per_env", "max_steps", "auto
           "ch_player", "ch_goal", "ch_empty", "ch_wall", "border_wall", "cum_per_env")
 
 
+class OrMutation(ctypes.Structure):
+    _fields_ = [("p_map", ctypes.c_uint32), ("map_channels", ctypes.c_uint32),
+                ("p_rule", ctypes.c_uint32), ("p_reward", ctypes.c_uint32),
+                ("reward_min", ctypes.c_int32), ("reward_max", ctypes.c_int32),
+                ("mutable_rules", ctypes.c_uint64)]
+
+
 class OrCfg(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int32) for f in FIELDS]
 
@@ -68,6 +75,8 @@ def lib():
         L.or_observe.argtypes = [vp, i32, vp, i32, vp, vp]
         L.or_rule_obs.restype = i32
         L.or_rule_obs.argtypes = [vp, vp, i32, vp, vp]
+        L.or_mutate.restype = i32
+        L.or_mutate.argtypes = [i32, vp, i32, i32, i32, i32, vp, u64, vp, vp]
         _lib = L
     return _lib
 
@@ -239,3 +248,21 @@ def rule_obs(cfg: OrCfg, rules):
     rc = lib().or_rule_obs(ctypes.byref(cfg), _p(rb), T, _p(bits), _p(rew))
     assert rc == 0, rc
     return bits, rew
+
+
+def mutate(H: int, W: int, C: int, mutation: dict, seed: int, maps=None, rules=None,
+           env_ids=None):
+    """Mutation operators of the evolution loop: returns mutated copies of
+    maps [n, H, W] and rule tables [n, R] (either may be None).  mutation:
+    p_map, map_channels, p_rule, p_reward (24-bit thresholds), reward_min,
+    reward_max, mutable_rules (bit mask over rule slots)."""
+    m = OrMutation(**{k: int(mutation[k]) for k, _ in OrMutation._fields_})
+    n = maps.shape[0] if maps is not None else rules.shape[0]
+    mp = None if maps is None else np.array(maps, dtype=cell_dtype(C), copy=True, order="C")
+    rl = None if rules is None else np.array(rules, copy=True, order="C")
+    R = 0 if rl is None else rl.shape[1]
+    rb = None if rl is None else rl.view(np.uint8).reshape(-1)
+    rc = lib().or_mutate(n, _p(_ids(env_ids, n)), H, W, C, R, ctypes.byref(m), int(seed) & (2**64 - 1),
+                         _p(mp), _p(rb))
+    assert rc == 0, rc
+    return mp, rl

@@ -891,3 +891,121 @@ int or_rule_obs(const or_cfg *cfg, const uint8_t *rules, int n_tables, uint8_t *
         }
     return 0;
 }
+
+/* ------------------------------------------------------------ mutation
+ * The mutation operators of the evolution loop (Sec. 3.1.1):
+ *  - the initial map, a multi-hot array, is mutated by flipping bits at
+ *    random (last paragraph);
+ *  - the mutable rules (the empty "no-op" rules added to the base game, not
+ *    the base game's own) are mutated by changing tiles of the input and/or
+ *    output pattern at various positions (first paragraph);
+ *  - a rule's reward may be changed as well, to positive or negative values
+ *    (second paragraph).
+ *
+ * Readings (the paper gives no rates, order or encoding):
+ *  - every decision is an independent Bernoulli draw from the counter RNG,
+ *    u = draw >> 40 (24 bits), taken when u < p (p in units of 2^-24);
+ *  - map: bit c of cell q = y*W + x of env b flips when
+ *    draw(seed, 9, b, q, c) >> 40 < p_map, for the channels in map_channels;
+ *  - rules: an input entry (rule r, pattern entry e < h*w, channel c <= C)
+ *    has three states, don't-care / present / absent, and an output entry
+ *    (channel c < C) three, unchanged / set / clear; with d =
+ *    draw(seed, 10 (input) or 11 (output), t, 25*r + e, c), the entry changes
+ *    when d >> 40 < p_rule, to the next state (cyclically) when bit 39 of d
+ *    is 0 and the one after it when 1 -- a change to one of the two other
+ *    states, each equally likely;
+ *  - reward: with d = draw(seed, 12, t, r, 0), when d >> 40 < p_reward the
+ *    reward becomes reward_min + ((draw(seed, 12, t, r, 1) >> 32) * n >> 32),
+ *    n = reward_max - reward_min + 1 (uniform, may equal the old one);
+ *  - only rules whose bit is set in mutable_rules change; the pattern size
+ *    h x w is kept.
+ * env_ids (nullable) give the global environment / table index used in the
+ * draws for each of the n maps and n tables passed. */
+typedef struct {
+    uint32_t p_map, map_channels, p_rule, p_reward;
+    int32_t reward_min, reward_max;
+    uint64_t mutable_rules;
+} or_mutation;
+
+static void wr32(uint8_t *p, uint32_t v)
+{
+    p[0] = (uint8_t)v;
+    p[1] = (uint8_t)(v >> 8);
+    p[2] = (uint8_t)(v >> 16);
+    p[3] = (uint8_t)(v >> 24);
+}
+
+/* Ternary state of bit c in a pair of masks (one, two): 0 neither, 1 one, 2 two. */
+static int tern_get(uint32_t one, uint32_t two, int c) { return ((one >> c) & 1u) ? 1 : ((two >> c) & 1u) ? 2 : 0; }
+
+static void tern_set(uint32_t *one, uint32_t *two, int c, int state)
+{
+    *one &= ~(1u << c);
+    *two &= ~(1u << c);
+    if (state == 1)
+        *one |= 1u << c;
+    else if (state == 2)
+        *two |= 1u << c;
+}
+
+static int mutated_state(uint64_t d, uint32_t p, int state)
+{
+    if ((uint32_t)(d >> 40) >= p)
+        return state;
+    return (state + 1 + (int)((d >> 39) & 1u)) % 3;
+}
+
+int or_mutate(int n, const int32_t *env_ids, int H, int W, int C, int R, const or_mutation *m,
+              uint64_t seed, void *maps, uint8_t *rules)
+{
+    if (n < 0 || H < 1 || W < 1 || H > OR_MAXSIDE || W > OR_MAXSIDE || C < 1 || C > 16 || R < 0 ||
+        R > 64)
+        return -1;
+    const size_t gb = (size_t)H * W * cell_bytes(C);
+    uint32_t cells[OR_MAXCELLS];
+    for (int i = 0; i < n; i++) {
+        const uint64_t b = env_ids ? (uint64_t)env_ids[i] : (uint64_t)i;
+        if (maps) {
+            uint8_t *g = (uint8_t *)maps + (size_t)i * gb;
+            load_grid(g, H, W, C, cells);
+            for (int q = 0; q < H * W; q++)
+                for (int c = 0; c < C; c++)
+                    if (((m->map_channels >> c) & 1u) && (uint32_t)(or_draw(seed, 9, b, q, c) >> 40) < m->p_map)
+                        cells[q] ^= 1u << c;
+            store_grid(cells, H, W, C, g);
+        }
+        if (!rules)
+            continue;
+        for (int r = 0; r < R; r++) {
+            if (!((m->mutable_rules >> r) & 1u))
+                continue;
+            uint8_t *rec = rules + ((size_t)i * R + r) * OR_RULE_BYTES;
+            or_pattern p;
+            parse_rule(rec, &p);
+            for (int e = 0; e < p.h * p.w; e++) {
+                for (int c = 0; c <= C; c++) {
+                    const uint64_t d = or_draw(seed, 10, b, 25u * r + e, c);
+                    tern_set(&p.present[e], &p.absent[e], c,
+                             mutated_state(d, m->p_rule, tern_get(p.present[e], p.absent[e], c)));
+                }
+                for (int c = 0; c < C; c++) {
+                    const uint64_t d = or_draw(seed, 11, b, 25u * r + e, c);
+                    tern_set(&p.set[e], &p.clear[e], c,
+                             mutated_state(d, m->p_rule, tern_get(p.set[e], p.clear[e], c)));
+                }
+            }
+            if ((uint32_t)(or_draw(seed, 12, b, r, 0) >> 40) < m->p_reward) {
+                const uint64_t span = (uint64_t)((int64_t)m->reward_max - m->reward_min + 1);
+                p.reward = (int32_t)(m->reward_min + (int64_t)(((or_draw(seed, 12, b, r, 1) >> 32) * span) >> 32));
+            }
+            wr32(rec + 4, (uint32_t)p.reward);
+            for (int e = 0; e < 25; e++) {
+                wr32(rec + 8 + 4 * e, p.present[e]);
+                wr32(rec + 108 + 4 * e, p.absent[e]);
+                wr32(rec + 208 + 4 * e, p.set[e]);
+                wr32(rec + 308 + 4 * e, p.clear[e]);
+            }
+        }
+    }
+    return 0;
+}
