@@ -866,6 +866,219 @@ def run_observe_reference(args, wl: ObserveWorkload):
     return 0
 
 
+# ------------------------------------------------------------- mutation
+MUTATE_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_mutate.cu")
+MIX64_OPS = 20  # 32-bit operations of one SplitMix64 finaliser (3 xor-shifts, 2 64-bit multiplies, input xor)
+
+
+class MutateName:
+    """Name of the mutation workload (for its profile summary)."""
+
+    def __init__(self, wl):
+        self.name = f"mutate-grid{wl.H}-b{wl.batch}-c{wl.C}-r{wl.n_rules}"
+
+
+def mutation_rates(wl) -> dict:
+    """Rates of the mutation benchmark: about ten map bits per board, one in
+    eight rule entries, one in four rewards; every rule slot mutable."""
+    bits = wl.H * wl.W * wl.C
+    return dict(p_map=max(1, (10 << 24) // bits), map_channels=(1 << wl.C) - 1, p_rule=1 << 21,
+                p_reward=1 << 22, reward_min=wl.reward_lo, reward_max=wl.reward_hi,
+                mutable_rules=(1 << wl.n_rules) - 1)
+
+
+def mutation_draws(wl, rules) -> float:
+    """Counter draws (one mix each) per environment of one av_mutate call,
+    averaged over the tables, plus the three-mix prefixes per stream."""
+    cells = wl.H * wl.W * wl.C + 2
+    entries = (rules["h"].astype(np.int64) * rules["w"]).sum(axis=1).mean()
+    rule_draws = entries * (2 * wl.C + 1) + 4 + 2 + wl.n_rules * (1 + 0.25)
+    return float(cells + rule_draws)
+
+
+def run_mutate(args, wl):
+    """One benchmark step = one av_mutate call over every map and rule table
+    of the 16,384-env training shape."""
+    import torch
+
+    import paper_2407_04221_gb300 as av
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    seed = args.seed + 1000 * rank
+    _, rules, cum = wk.make(wl, seed)
+    fields = wk.config_fields(wl)
+    import oracle
+    cfg = oracle.make_cfg(**fields)
+    env = av.Env(fields, rules, cum, device=dev)
+    maps0 = env.reset(wk.seeds(seed)["reset"])
+    env.close()
+    B, R = wl.batch, wl.n_rules
+    maps = maps0.clone()
+    rules_dev = torch.from_numpy(np.ascontiguousarray(rules).view(np.uint8).reshape(B, R, 408).copy()).to(dev)
+    rates = mutation_rates(wl)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+
+    def launch(i):
+        av.av_mutate(B, wl.H, wl.W, wl.C, R, rates, seed * 7919 + i, maps, rules_dev, stream)
+
+    for i in range(args.warmup):
+        launch(i)
+    torch.cuda.synchronize(dev)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(torch.cuda.current_device() if world == 1 else local)
+    sampler.start()
+    barrier()
+    sampler.mark_start()
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.fill_(i & 0xff)
+        starts[i].record(stream)
+        launch(args.warmup + i)
+        ends[i].record(stream)
+    barrier()
+    wall = time.perf_counter() - t_wall
+    sampler.mark_end()
+    clocks = sampler.stop()
+    ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
+    kernel_ms = sum(ms) / len(ms)
+    total_ms = max_over_ranks(sum(ms), world, dev)
+    value = B * args.steps * world / (total_ms / 1e3)
+
+    # ---- e2e: maps and tables from pinned host memory, mutated copies back
+    h_maps = maps0.cpu().pin_memory()
+    h_rules = rules_dev.cpu().pin_memory()
+    o_maps = torch.empty_like(h_maps).pin_memory()
+    o_rules = torch.empty_like(h_rules).pin_memory()
+    e2e_steps = max(3, min(args.steps, 20))
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_steps):
+        maps.copy_(h_maps, non_blocking=True)
+        rules_dev.copy_(h_rules, non_blocking=True)
+        launch(50_000 + i)
+        o_maps.copy_(maps, non_blocking=True)
+        o_rules.copy_(rules_dev, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
+    e2e_value = B * world / (e2e_ms / 1e3)
+
+    if rank == 0:
+        peaks = measured_peaks()
+        sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+        peak_ops = SM_COUNT_GB300 * INT_LANES_PER_SM * sm_max * 1e6 / 1e9
+        ops = mutation_draws(wl, rules) * MIX64_OPS
+        achieved = ops * B / (kernel_ms / 1e3) / 1e9
+        nbytes = 2 * (wl.H * wl.W * wl.cell_bytes + R * 408)
+        hbm = float(peaks.get("hbm_gbs", 6800.0))
+        line = {
+            "metric": "env-mutations/s", "value": value, "unit": "env-mutations/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+            "config": {"workload": MutateName(wl).name, "batch": B, "H": wl.H,
+                       "W": wl.W, "tile_channels": wl.C, "rules": R, "rates": rates,
+                       "l2": "flushed (256 MiB write) between timed launches",
+                       "parallelism": "replicas"},
+            "e2e": {"value": e2e_value, "unit": "env-mutations/s",
+                    "h2d_bytes_per_step": int(h_maps.numel() * h_maps.element_size() + h_rules.numel()),
+                    "d2h_bytes_per_step": int(o_maps.numel() * o_maps.element_size() + o_rules.numel())},
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": peak_ops, "unit": "Gop/s",
+                         "frac": achieved / peak_ops,
+                         "traffic": profile_traffic("mutate_kernels", MutateName(wl), MUTATE_SRC),
+                         "kernel": "mutate_maps_kernel + mutate_rules_kernel",
+                         "ops_per_env": ops,
+                         "ops_basis": f"one SplitMix64 mix ({MIX64_OPS} 32-bit ops) per decision"
+                                      " (map bit, rule entry channel, reward) plus the per-stream"
+                                      " prefixes",
+                         "hbm_frac": nbytes * B / (kernel_ms / 1e3) / 1e9 / hbm,
+                         "bytes_per_env": nbytes,
+                         "peak_from": f"{SM_COUNT_GB300} SMs x {INT_LANES_PER_SM} int32 lanes/clk"
+                                      f" x {sm_max:.0f} MHz (sm_max_mhz of measured peaks)"},
+            "gpu_launches": 2 * args.steps,
+            "wall_s_timed_region": wall,
+        }
+        if clocks:
+            line["clocks"] = clocks
+        if world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = mutate_cpu_baseline(wl, rules, maps0, rates, seed)
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def mutate_cpu_baseline(wl, rules, maps0, rates, seed, budget_s: float = 3.0) -> dict:
+    """The oracle's mutation, one thread, on a sample of environments."""
+    import oracle
+    m = maps0.cpu().numpy()
+    m = m.view(np.uint16) if m.dtype == np.int16 else m
+    n = 256
+    ids = np.arange(n, dtype=np.int32)
+    reps, t0 = 0, time.perf_counter()
+    while True:
+        oracle.mutate(wl.H, wl.W, wl.C, rates, seed, m[:n], rules[:n], env_ids=ids)
+        reps += 1
+        dt = time.perf_counter() - t0
+        if dt > budget_s:
+            break
+    return {"value": reps * n / dt, "unit": "env-mutations/s", "cores": 1, "kind": "oracle",
+            "sample": f"{n} of {wl.batch} envs x {reps} passes", "seconds": dt}
+
+
+def run_mutate_reference(args, wl):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    _, rules, cum = wk.make(wl, args.seed)
+    cfg = oracle.make_cfg(**wk.config_fields(wl))
+    n = 1024
+    maps = oracle.reset(cfg, cum, wk.seeds(args.seed)["reset"], range(n))
+    rates = mutation_rates(wl)
+    ids = np.arange(n, dtype=np.int32)
+    for _ in range(args.warmup):
+        oracle.mutate(wl.H, wl.W, wl.C, rates, 1, maps[:64], rules[:64], env_ids=ids[:64])
+    times = []
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.mutate(wl.H, wl.W, wl.C, rates, i, maps, rules[:n], env_ids=ids)
+        times.append(time.perf_counter() - t0)
+    mean = sum(times) / len(times)
+    value = n / mean
+    line = {
+        "impl": "reference", "metric": "env-mutations/s", "value": value,
+        "unit": "env-mutations/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": mean * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+        "config": {"workload": f"mutate-grid{wl.H}-b{wl.batch}-c{wl.C}-r{wl.n_rules}",
+                   "sample_envs": n, "rates": rates},
+        "cpu_baseline": {"value": value, "unit": "env-mutations/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{n} of {wl.batch} envs per step"},
+        "e2e": {"value": value, "unit": "env-mutations/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
 def run_int_probe() -> int:
     """Build and run the integer-issue probe (needs nvcc and a GPU)."""
     import tempfile
@@ -894,11 +1107,18 @@ def main(argv=None):
     ap.add_argument("--observe", type=int, default=0, metavar="WINDOW",
                     help="time av_observe (player-centred patches of this width) on the"
                          " 16,384-env training shape instead of a rollout")
+    ap.add_argument("--mutate", action="store_true",
+                    help="time av_mutate (maps and rule tables) on the 16,384-env training shape")
     args = ap.parse_args(argv)
     if args.int_probe:
         return run_int_probe()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.mutate:
+        base = workload_for(3)
+        if args.batch > 0:
+            base = base.scaled(batch=args.batch)
+        return run_mutate_reference(args, base) if args.impl == "reference" else run_mutate(args, base)
     if args.observe:
         base = workload_for(3)
         if args.batch > 0:

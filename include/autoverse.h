@@ -186,6 +186,42 @@ int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, in
  * AV_EINVAL for a NULL bits with R > 0. */
 int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream);
 
+/* Rates and ranges of the mutation operators (av_mutate). */
+typedef struct {
+    uint32_t p_map;         /* map bit flip rate x 2^24 (0..2^24)                       */
+    uint32_t map_channels;  /* bit c: tile channel c of the maps may flip               */
+    uint32_t p_rule;        /* rule entry change rate x 2^24 (0..2^24)                  */
+    uint32_t p_reward;      /* reward redraw rate x 2^24 (0..2^24)                      */
+    int32_t reward_min, reward_max; /* redrawn rewards are uniform in [min, max]        */
+    uint64_t mutable_rules; /* bit r: rule slot r of every table may mutate             */
+} av_mutation;
+
+/* Mutation operators of the evolution loop (Sec. 3.1.1: the initial map, a
+ * multi-hot array, is mutated by flipping bits; the mutable rules by changing
+ * tiles of their input and/or output patterns at any position; rewards may
+ * change too, to positive or negative values).  In place, on caller-owned
+ * device arrays, without a handle:
+ *   maps:  device [batch][H][W] cell words (uint8 when C <= 8, else uint16),
+ *          or NULL: bit c of cell q = y*W + x of env b flips when
+ *          draw(seed, 9, b, q, c) >> 40 < p_map and bit c of map_channels is set;
+ *   rules: device av_rule [batch][n_rules], or NULL: for every rule slot r in
+ *          mutable_rules, every entry e < h*w of the input pattern (channels
+ *          0..C, force included; states don't-care / present / absent) and
+ *          of the output pattern (channels 0..C-1; states unchanged / set /
+ *          clear) changes when d >> 40 < p_rule, d = draw(seed, 10 (input) or
+ *          11 (output), b, 25 r + e, c), to the next state cyclically when
+ *          bit 39 of d is 0, else to the one after; the reward becomes
+ *          reward_min + ((draw(seed, 12, b, r, 1) >> 32) * n >> 32),
+ *          n = reward_max - reward_min + 1, when draw(seed, 12, b, r, 0) >> 40
+ *          < p_reward.  Pattern sizes do not change.
+ * draw is the counter draw of av_rollout.  Records must be valid (as av_create
+ * checks); mutated records stay valid.  A new handle made from the mutated
+ * records (av_create, host copies) and maps (av_set_state with set_as_init)
+ * evaluates the offspring.  AV_EINVAL for sizes outside the av_config limits,
+ * a NULL m, a rate above 2^24 or reward_min > reward_max. */
+int av_mutate(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t n_rules, const av_mutation *m,
+              uint64_t seed, void *maps, av_rule *rules, uintptr_t stream);
+
 /* Start a search from the root boards roots (device [B][H][W]): writes
  * root_hash uint64[B] (FNV-1a 64 as in av_expand) and root_live uint8[B]
  * (1 unless the root has no goal left), and sets the visited set of env b

@@ -24,7 +24,7 @@ AV_PATH_BLOCK, AV_PATH_FAST, AV_PATH_WARP = 1, 2, 3
 RULE_BYTES = 408
 EXPORTS = ("av_create", "av_destroy", "av_reset", "av_set_state", "av_get_state", "av_step",
            "av_rollout", "av_expand", "av_search_init", "av_select", "av_select_static", "av_sync",
-           "av_warnings", "av_rollout_path", "av_observe", "av_rule_obs", "av_strerror",
+           "av_warnings", "av_rollout_path", "av_observe", "av_rule_obs", "av_mutate", "av_strerror",
            "av_last_error")
 AV_MAX_WINDOW = 127
 AV_SELECT_STATIC_MAX_HASHES = 1 << 21
@@ -39,6 +39,13 @@ class AvConfig(ctypes.Structure):
                 ("ch_wall", ctypes.c_int32), ("border_wall", ctypes.c_int32),
                 ("cum_per_env", ctypes.c_int32), ("init_cum", ctypes.c_void_p),
                 ("search_capacity", ctypes.c_int32)]
+
+
+class AvMutation(ctypes.Structure):
+    _fields_ = [("p_map", ctypes.c_uint32), ("map_channels", ctypes.c_uint32),
+                ("p_rule", ctypes.c_uint32), ("p_reward", ctypes.c_uint32),
+                ("reward_min", ctypes.c_int32), ("reward_max", ctypes.c_int32),
+                ("mutable_rules", ctypes.c_uint64)]
 
 
 class AvError(RuntimeError):
@@ -78,6 +85,7 @@ def load() -> ctypes.CDLL:
         "av_rollout_path": [vp, ctypes.POINTER(ctypes.c_int32)],
         "av_observe": [vp, vp, i32, vp, vp, up],
         "av_rule_obs": [vp, vp, vp, up],
+        "av_mutate": [i32, i32, i32, i32, i32, ctypes.POINTER(AvMutation), u64, vp, vp, up],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -239,6 +247,18 @@ def av_observe(h, grids, window: int, obs, player_yx=None, stream=None):
 def av_rule_obs(h, bits, reward=None, stream=None):
     """Binary form of the rule tables: bits [T, R, 4, 5, 5, C+1] uint8, reward [T, R]."""
     _check(h, "av_rule_obs", load().av_rule_obs(h, _ptr(bits), _ptr(reward), _stream(stream)))
+
+
+def av_mutate(batch, H, W, C, n_rules, mutation: dict, seed: int, maps=None, rules=None,
+              stream=None):
+    """Mutation operators (Sec. 3.1.1), in place on device tensors: maps
+    [batch, H, W] cell words, rules [batch, n_rules, 408] uint8 packed records
+    (either may be None).  mutation: p_map, map_channels, p_rule, p_reward
+    (rates x 2^24), reward_min, reward_max, mutable_rules (bit mask)."""
+    m = AvMutation(**{k: int(mutation[k]) for k, _ in AvMutation._fields_})
+    rc = load().av_mutate(int(batch), int(H), int(W), int(C), int(n_rules), ctypes.byref(m),
+                          int(seed) & (2**64 - 1), _ptr(maps), _ptr(rules), _stream(stream))
+    _check(None, "av_mutate", rc)
 
 
 class Env:

@@ -673,6 +673,22 @@ int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream)
     return launch_check(h, "rule observation kernel");
 }
 
+int av_mutate(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t n_rules, const av_mutation *m,
+              uint64_t seed, void *maps, av_rule *rules, uintptr_t stream)
+{
+    if (!m || batch < 1 || H < 1 || H > AV_MAX_SIDE || W < 1 || W > AV_MAX_SIDE || C < 1 || C > AV_MAX_C ||
+        n_rules < 0 || n_rules > AV_MAX_RULES)
+        return AV_EINVAL;
+    const uint32_t one = 1u << 24;
+    if (m->p_map > one || m->p_rule > one || m->p_reward > one || m->reward_min > m->reward_max)
+        return AV_EINVAL;
+    launch_mutate(batch, H, W, C, n_rules, m->p_map, m->map_channels, m->p_rule, m->p_reward, m->reward_min,
+                  m->reward_max, m->mutable_rules, seed, maps, reinterpret_cast<uint32_t *>(rules),
+                  as_stream(stream));
+    const cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? AV_OK : AV_ECUDA;
+}
+
 int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t *root_live,
                    uintptr_t stream)
 {

@@ -72,6 +72,11 @@ void launch_observe(const DevConfig &cf, const void *grids, int window, uint8_t 
 void launch_rule_obs(int n_rules_total, int C, const uint32_t *rules, uint8_t *bits, int32_t *reward,
                      cudaStream_t st);
 
+// Mutation operators (k_mutate.cu).
+void launch_mutate(int B, int H, int W, int C, int R, uint32_t p_map, uint32_t map_channels, uint32_t p_rule,
+                   uint32_t p_reward, int32_t reward_min, int32_t reward_max, uint64_t mutable_rules, uint64_t seed,
+                   void *maps, uint32_t *rules, cudaStream_t st);
+
 inline cudaError_t configure_kernels()
 {
     cudaError_t e = configure_fast_u8();

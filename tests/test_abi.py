@@ -60,6 +60,13 @@ def test_host_side_argument_checks(lib):
     assert lib.av_rollout_path(None, None) == av.AV_EINVAL
     assert lib.av_observe(None, None, 5, None, None, 0) == av.AV_EINVAL
     assert lib.av_rule_obs(None, None, None, 0) == av.AV_EINVAL
+    assert lib.av_mutate(1, 16, 16, 8, 8, None, 0, None, None, 0) == av.AV_EINVAL
+    m = av.AvMutation(p_map=(1 << 24) + 1)
+    assert lib.av_mutate(1, 16, 16, 8, 8, ctypes.byref(m), 0, None, None, 0) == av.AV_EINVAL
+    m = av.AvMutation(reward_min=2, reward_max=1)
+    assert lib.av_mutate(1, 16, 16, 8, 8, ctypes.byref(m), 0, None, None, 0) == av.AV_EINVAL
+    m = av.AvMutation()
+    assert lib.av_mutate(1, 65, 16, 8, 8, ctypes.byref(m), 0, None, None, 0) == av.AV_EINVAL
     assert av.av_strerror(av.AV_EINVAL) == "invalid argument"
     base = dict(batch=1, H=16, W=16, C=4, n_rules=0, rules_per_env=0, max_steps=0, auto_reset=0,
                 ch_player=2, ch_goal=3, ch_empty=0, ch_wall=1, border_wall=1, cum_per_env=0)
