@@ -24,6 +24,25 @@ FIELDS = ("batch", "H", "W", "C", "n_rules", "rules_per_env", "max_steps", "auto
           "ch_player", "ch_goal", "ch_empty", "ch_wall", "border_wall", "cum_per_env")
 
 
+class OrVariant(ctypes.Structure):
+    _fields_ = [("random_keys", ctypes.c_int32), ("_pad", ctypes.c_int32),
+                ("key_seed", ctypes.c_uint64), ("limit", ctypes.c_int32 * 64),
+                ("inhibit", ctypes.c_uint64 * 64)]
+
+
+def make_variant(random_keys=0, key_seed=0, limit=None, inhibit=None) -> OrVariant:
+    """Variant semantics: limit[r] matches per step (0 = all) chosen by
+    largest key, inhibit[r] = bit mask of the rules a match of r suppresses."""
+    v = OrVariant()
+    v.random_keys = int(random_keys)
+    v.key_seed = int(key_seed) & (2**64 - 1)
+    for r, k in enumerate(limit or []):
+        v.limit[r] = int(k)
+    for r, m in enumerate(inhibit or []):
+        v.inhibit[r] = int(m)
+    return v
+
+
 class OrMutation(ctypes.Structure):
     _fields_ = [("p_map", ctypes.c_uint32), ("map_channels", ctypes.c_uint32),
                 ("p_rule", ctypes.c_uint32), ("p_reward", ctypes.c_uint32),
@@ -75,6 +94,10 @@ def lib():
         L.or_observe.argtypes = [vp, i32, vp, i32, vp, vp]
         L.or_rule_obs.restype = i32
         L.or_rule_obs.argtypes = [vp, vp, i32, vp, vp]
+        L.or_step_batch_v.restype = i32
+        L.or_step_batch_v.argtypes = [vp, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32]
+        L.or_rollout_v.restype = i32
+        L.or_rollout_v.argtypes = [vp, vp, vp, i32, vp, vp, vp, vp, i32, u64, vp, vp, vp, vp, i32]
         L.or_mutate.restype = i32
         L.or_mutate.argtypes = [i32, vp, i32, i32, i32, i32, vp, u64, vp, vp]
         _lib = L
@@ -145,8 +168,8 @@ def reset(cfg: OrCfg, cum: np.ndarray, seed: int, envs) -> np.ndarray:
     return out
 
 
-def step(cfg: OrCfg, rules, grids, inits, t, actions, env_ids=None, threads=None):
-    """One step of n envs -> (grids, t, rewards, dones)."""
+def step(cfg: OrCfg, rules, grids, inits, t, actions, env_ids=None, threads=None, variant=None):
+    """One step of n envs -> (grids, t, rewards, dones); variant: OrVariant or None."""
     grids = np.ascontiguousarray(grids, dtype=cell_dtype(cfg.C))
     n = grids.shape[0]
     inits = np.ascontiguousarray(inits, dtype=cell_dtype(cfg.C))
@@ -158,15 +181,15 @@ def step(cfg: OrCfg, rules, grids, inits, t, actions, env_ids=None, threads=None
     done = np.zeros(n, np.uint8)
     rb = _rules_buf(rules)
     ids = _ids(env_ids, n)
-    rc = lib().or_step_batch(ctypes.byref(cfg), _p(rb), n, _p(ids), _p(grids), _p(inits), _p(t),
-                             _p(actions), _p(out), _p(t_out), _p(rew), _p(done),
-                             threads or default_threads())
+    rc = lib().or_step_batch_v(ctypes.byref(cfg), _p(rb), None if variant is None else ctypes.byref(variant),
+                               n, _p(ids), _p(grids), _p(inits), _p(t), _p(actions), _p(out),
+                               _p(t_out), _p(rew), _p(done), threads or default_threads())
     assert rc == 0, rc
     return out, t_out, rew, done
 
 
 def rollout(cfg: OrCfg, rules, grids, inits, t, n_steps, action_seed, env_ids=None,
-            trajectory=False, threads=None):
+            trajectory=False, threads=None, variant=None):
     """Fused rollout -> dict(grids, t, rew_sum[, obs, rew, done])."""
     grids = np.array(grids, dtype=cell_dtype(cfg.C), copy=True, order="C")
     n = grids.shape[0]
@@ -180,9 +203,9 @@ def rollout(cfg: OrCfg, rules, grids, inits, t, n_steps, action_seed, env_ids=No
         done = np.zeros((n_steps, n), np.uint8)
     rb = _rules_buf(rules)
     ids = _ids(env_ids, n)
-    rc = lib().or_rollout(ctypes.byref(cfg), _p(rb), n, _p(ids), _p(grids), _p(inits), _p(t),
-                          int(n_steps), int(action_seed), _p(obs), _p(rew), _p(done), _p(rew_sum),
-                          threads or default_threads())
+    rc = lib().or_rollout_v(ctypes.byref(cfg), _p(rb), None if variant is None else ctypes.byref(variant),
+                            n, _p(ids), _p(grids), _p(inits), _p(t), int(n_steps), int(action_seed),
+                            _p(obs), _p(rew), _p(done), _p(rew_sum), threads or default_threads())
     assert rc == 0, rc
     res = dict(grids=grids, t=t, rew_sum=rew_sum)
     if trajectory:

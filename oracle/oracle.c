@@ -309,6 +309,142 @@ static void transition(const or_cfg *cfg, const or_rules *rs, const uint32_t *G,
     *reward = rew;
 }
 
+/* ----------------------------------------------------- variant semantics
+ * The possible extensions at the end of Sec. 2.1: a rule may be applied only
+ * once or a fixed number of times per step, the tiles to rewrite chosen by
+ * taking the maximum over an additional channel of ordered or random index
+ * values; and masking may let certain rules inhibit others.
+ *
+ * Readings (the paper only sketches them):
+ *  - a match is (rule r, rotation j, anchor cell q = y0*W + x0); its key is
+ *    (q << 2) | j with ordered indices, or ((draw(key_seed, 13, env, t, q)
+ *    >> 48) << 14) | (q << 2) | j with random ones (t: the env's step counter
+ *    before the step), so every match of a rule has a distinct key;
+ *  - limit[r] = k > 0: of rule r's matches this step only the k with the
+ *    largest keys apply (write and pay); 0: all apply;
+ *  - inhibit[r]: when rule r has at least one match this step (before any
+ *    limit or inhibition), every rule s with bit s of inhibit[r] set is
+ *    suppressed this step (no writes, no reward) -- decided on raw matches,
+ *    so the result does not depend on rule order. */
+typedef struct {
+    int32_t random_keys;
+    int32_t _pad;
+    uint64_t key_seed;
+    int32_t limit[64];
+    uint64_t inhibit[64];
+} or_variant;
+
+typedef struct {
+    uint32_t key;
+    int16_t j, y0, x0;
+} or_match;
+
+static int cmp_match_desc(const void *a, const void *b)
+{
+    uint32_t ka = ((const or_match *)a)->key, kb = ((const or_match *)b)->key;
+    return ka < kb ? 1 : ka > kb ? -1 : 0;
+}
+
+static void transition_variant(const or_cfg *cfg, const or_rules *rs, const or_variant *v, uint64_t env,
+                               int32_t t, const uint32_t *G, int action, uint32_t *N, int32_t *reward,
+                               or_match *buf)
+{
+    const int H = cfg->H, W = cfg->W, C = cfg->C;
+    uint32_t F[OR_MAXCELLS], SETm[OR_MAXCELLS], CLRm[OR_MAXCELLS];
+    int32_t rew = 0;
+    for (int p = 0; p < H * W; p++)
+        F[p] = G[p];
+    if (action < 0 || action > 4)
+        action = 0;
+    if (cfg->ch_player >= 0 && action != 0)
+        for (int y = 0; y < H; y++)
+            for (int x = 0; x < W; x++) {
+                if (!((G[y * W + x] >> cfg->ch_player) & 1u))
+                    continue;
+                int yy = y + DY[action], xx = x + DX[action];
+                if (yy >= 0 && yy < H && xx >= 0 && xx < W)
+                    F[yy * W + xx] |= 1u << C;
+            }
+    for (int p = 0; p < H * W; p++)
+        SETm[p] = CLRm[p] = 0;
+
+    /* raw matches of every rule, before limits and inhibition */
+    int count[64];
+    int start[65];
+    start[0] = 0;
+    for (int r = 0; r < rs->R; r++) {
+        int n = 0;
+        for (int j = 0; j < 4; j++) {
+            const or_pattern *P = &rs->rot[4 * r + j];
+            for (int y0 = 0; y0 + P->h <= H; y0++)
+                for (int x0 = 0; x0 + P->w <= W; x0++) {
+                    int ok = 1;
+                    for (int i = 0; i < P->h && ok; i++)
+                        for (int k = 0; k < P->w && ok; k++) {
+                            uint32_t cell = F[(y0 + i) * W + (x0 + k)];
+                            int e = i * P->w + k;
+                            for (int c = 0; c <= C && ok; c++) {
+                                uint32_t bit = (cell >> c) & 1u;
+                                if (((P->present[e] >> c) & 1u) && !bit)
+                                    ok = 0;
+                                if (((P->absent[e] >> c) & 1u) && bit)
+                                    ok = 0;
+                            }
+                        }
+                    if (!ok)
+                        continue;
+                    const uint32_t q = (uint32_t)(y0 * W + x0);
+                    uint32_t key = (q << 2) | (uint32_t)j;
+                    if (v->random_keys)
+                        key |= (uint32_t)(or_draw(v->key_seed, 13, env, (uint64_t)(uint32_t)t, q) >> 48) << 14;
+                    or_match *m = &buf[start[r] + n++];
+                    m->key = key;
+                    m->j = (int16_t)j;
+                    m->y0 = (int16_t)y0;
+                    m->x0 = (int16_t)x0;
+                }
+        }
+        count[r] = n;
+        start[r + 1] = start[r] + n;
+    }
+    /* inhibition, from raw matches */
+    uint64_t suppressed = 0;
+    for (int r = 0; r < rs->R; r++)
+        if (count[r] > 0)
+            suppressed |= v->inhibit[r];
+    /* the applied matches: all, or the limit[r] with the largest keys */
+    for (int r = 0; r < rs->R; r++) {
+        if ((suppressed >> r) & 1u)
+            continue;
+        or_match *list = &buf[start[r]];
+        int n = count[r];
+        if (v->limit[r] > 0 && n > v->limit[r]) {
+            qsort(list, (size_t)n, sizeof(or_match), cmp_match_desc);
+            n = v->limit[r];
+        }
+        for (int m = 0; m < n; m++) {
+            const or_pattern *P = &rs->rot[4 * r + list[m].j];
+            rew += P->reward;
+            for (int i = 0; i < P->h; i++)
+                for (int k = 0; k < P->w; k++) {
+                    int e = i * P->w + k;
+                    SETm[(list[m].y0 + i) * W + (list[m].x0 + k)] |= P->set[e];
+                    CLRm[(list[m].y0 + i) * W + (list[m].x0 + k)] |= P->clear[e];
+                }
+        }
+    }
+    uint32_t tiles = (1u << C) - 1u;
+    for (int p = 0; p < H * W; p++)
+        N[p] = ((F[p] & ~CLRm[p]) | (~F[p] & SETm[p])) & tiles;
+    *reward = rew;
+}
+
+/* Room for every raw match of one step: 4 rotations x H*W anchors x R rules. */
+static or_match *match_buffer(const or_cfg *cfg)
+{
+    return (or_match *)malloc(sizeof(or_match) * 4 * (size_t)cfg->H * cfg->W * (cfg->n_rules > 0 ? cfg->n_rules : 1));
+}
+
 static int goal_left(const or_cfg *cfg, const uint32_t *N)
 {
     if (cfg->ch_goal < 0)
@@ -473,6 +609,7 @@ typedef struct {
     uint8_t *grids_out;
     int32_t *t_out, *rewards;
     uint8_t *dones;
+    const or_variant *v; /* NULL: standard semantics */
 } step_job;
 
 static int step_item(void *ctx, int n)
@@ -492,7 +629,17 @@ static int step_item(void *ctx, int n)
     load_grid(j->grids_in + gb * n, cfg->H, cfg->W, cfg->C, G);
     load_grid(j->inits + gb * n, cfg->H, cfg->W, cfg->C, I);
     int32_t rew, t = j->t_in[n];
-    transition(cfg, rs, G, j->actions[n], N, &rew);
+    if (j->v) {
+        or_match *buf = match_buffer(cfg);
+        if (!buf) {
+            free(rs);
+            return -2;
+        }
+        transition_variant(cfg, rs, j->v, (uint64_t)env, t, G, j->actions[n], N, &rew, buf);
+        free(buf);
+    } else {
+        transition(cfg, rs, G, j->actions[n], N, &rew);
+    }
     j->dones[n] = finish(cfg, N, I, &t);
     j->rewards[n] = rew;
     j->t_out[n] = t;
@@ -503,16 +650,25 @@ static int step_item(void *ctx, int n)
 
 /* One step of n envs.  env_ids (nullable) maps item n to the env index that
  * selects its rule table; grids are canonical [n][H][W] cell words. */
+int or_step_batch_v(const or_cfg *cfg, const uint8_t *rules, const or_variant *v, int n,
+                    const int32_t *env_ids, const void *grids_in, const void *inits,
+                    const int32_t *t_in, const uint8_t *actions, void *grids_out, int32_t *t_out,
+                    int32_t *rewards, uint8_t *dones, int threads)
+{
+    if (check_cfg(cfg))
+        return -1;
+    step_job j = {cfg, rules, env_ids, (const uint8_t *)grids_in, (const uint8_t *)inits, t_in,
+                  actions, (uint8_t *)grids_out, t_out, rewards, dones, v};
+    return run_pool(n, threads, &j, step_item);
+}
+
 int or_step_batch(const or_cfg *cfg, const uint8_t *rules, int n, const int32_t *env_ids,
                   const void *grids_in, const void *inits, const int32_t *t_in,
                   const uint8_t *actions, void *grids_out, int32_t *t_out, int32_t *rewards,
                   uint8_t *dones, int threads)
 {
-    if (check_cfg(cfg))
-        return -1;
-    step_job j = {cfg, rules, env_ids, (const uint8_t *)grids_in, (const uint8_t *)inits, t_in,
-                  actions, (uint8_t *)grids_out, t_out, rewards, dones};
-    return run_pool(n, threads, &j, step_item);
+    return or_step_batch_v(cfg, rules, NULL, n, env_ids, grids_in, inits, t_in, actions, grids_out,
+                           t_out, rewards, dones, threads);
 }
 
 /* -------------------------------------------------------------- rollout */
@@ -529,6 +685,7 @@ typedef struct {
     int32_t *rew_traj;
     uint8_t *done_traj;
     int32_t *rew_sum;
+    const or_variant *v; /* NULL: standard semantics */
 } roll_job;
 
 static int roll_item(void *ctx, int n)
@@ -548,10 +705,18 @@ static int roll_item(void *ctx, int n)
     load_grid(j->grids + gb * n, cfg->H, cfg->W, cfg->C, G);
     load_grid(j->inits + gb * n, cfg->H, cfg->W, cfg->C, I);
     int32_t t = j->t[n], sum = 0;
+    or_match *buf = NULL;
+    if (j->v && !(buf = match_buffer(cfg))) {
+        free(rs);
+        return -2;
+    }
     for (int s = 0; s < j->n_steps; s++) {
         int a = (int)uniform_below(or_draw(j->action_seed, 4, (uint64_t)env, 0, (uint64_t)s), 5);
         int32_t rew;
-        transition(cfg, rs, G, a, N, &rew);
+        if (j->v)
+            transition_variant(cfg, rs, j->v, (uint64_t)env, t, G, a, N, &rew, buf);
+        else
+            transition(cfg, rs, G, a, N, &rew);
         uint8_t d = finish(cfg, N, I, &t);
         sum += rew;
         size_t slot = (size_t)s * j->n + n;
@@ -567,6 +732,7 @@ static int roll_item(void *ctx, int n)
     j->t[n] = t;
     if (j->rew_sum)
         j->rew_sum[n] = sum;
+    free(buf);
     free(rs);
     return 0;
 }
@@ -574,15 +740,24 @@ static int roll_item(void *ctx, int n)
 /* n_steps fused steps of n envs with on-the-fly actions
  * a = uniform5(draw(action_seed, 4, env, 0, s)).  grids and t are updated in
  * place; trajectories are [n_steps][n] (nullable). */
-int or_rollout(const or_cfg *cfg, const uint8_t *rules, int n, const int32_t *env_ids, void *grids,
-               const void *inits, int32_t *t, int n_steps, uint64_t action_seed, void *obs_traj,
-               int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, int threads)
+int or_rollout_v(const or_cfg *cfg, const uint8_t *rules, const or_variant *v, int n,
+                 const int32_t *env_ids, void *grids, const void *inits, int32_t *t, int n_steps,
+                 uint64_t action_seed, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj,
+                 int32_t *rew_sum, int threads)
 {
     if (check_cfg(cfg) || n_steps < 0)
         return -1;
     roll_job j = {cfg, rules, env_ids, n, n_steps, action_seed, (uint8_t *)grids,
-                  (const uint8_t *)inits, t, (uint8_t *)obs_traj, rew_traj, done_traj, rew_sum};
+                  (const uint8_t *)inits, t, (uint8_t *)obs_traj, rew_traj, done_traj, rew_sum, v};
     return run_pool(n, threads, &j, roll_item);
+}
+
+int or_rollout(const or_cfg *cfg, const uint8_t *rules, int n, const int32_t *env_ids, void *grids,
+               const void *inits, int32_t *t, int n_steps, uint64_t action_seed, void *obs_traj,
+               int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, int threads)
+{
+    return or_rollout_v(cfg, rules, NULL, n, env_ids, grids, inits, t, n_steps, action_seed,
+                        obs_traj, rew_traj, done_traj, rew_sum, threads);
 }
 
 /* --------------------------------------------------------------- expand */

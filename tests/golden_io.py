@@ -5,7 +5,8 @@ Fixture format (one step of one env):
     # comment lines; a '# cite:' line names the passage the case follows
     channels: E W P G          names of tile channels 0..C-1 (force is 'F')
     roles: player=P goal=G empty=E wall=W
-    rule <name> reward=<int> size=<h>x<w>
+    rule <name> reward=<int> size=<h>x<w>  (variant fixtures add 'limit: <rule> <k>',
+                               'inhibit: <rule> <rule>', 'index: ordered|random')
     in:
       <h lines of w entries>   entry: letters = present channels, '!X' = X absent,
                                'F' = force present, '.' = don't care
@@ -45,6 +46,7 @@ class Fixture:
     after: np.ndarray
     reward: int
     done: int
+    variant: dict = dataclasses.field(default_factory=dict)  # limit {r: k}, inhibit {r: mask}, index
 
     def cfg_fields(self) -> dict:
         H, W = self.before.shape
@@ -95,6 +97,7 @@ def load(path: str) -> Fixture:
     cite = " ".join(ln.split(":", 1)[1].strip() for ln in lines if ln.startswith("# cite:"))
     body = [ln.strip() for ln in lines if ln.strip() and not ln.startswith("#")]
     names, roles, rules = {}, {}, []
+    variant = {"limit": {}, "inhibit": {}, "index": "ordered"}
     action = reward = done = 0
     before = after = None
     i = 0
@@ -141,6 +144,17 @@ def load(path: str) -> Fixture:
             assert body[i + 3 + 2 * h] == "end"
             rules.append(rec)
             i += 4 + 2 * h
+        elif ln.startswith("limit:"):
+            r, k = (int(v) for v in ln.split(":")[1].split())
+            variant["limit"][r] = k
+            i += 1
+        elif ln.startswith("inhibit:"):
+            r, q = (int(v) for v in ln.split(":")[1].split())
+            variant["inhibit"][r] = variant["inhibit"].get(r, 0) | (1 << q)
+            i += 1
+        elif ln.startswith("index:"):
+            variant["index"] = ln.split(":")[1].strip()
+            i += 1
         elif ln.startswith("action:"):
             action = int(ln.split(":")[1])
             i += 1
@@ -166,7 +180,12 @@ def load(path: str) -> Fixture:
     for r, rec in enumerate(rules):
         rt[0, r] = rec
     return Fixture(os.path.basename(path), cite, C, roles, rt, action, before.astype(dt),
-                   after.astype(dt), reward, done)
+                   after.astype(dt), reward, done, variant)
+
+
+def variant_fixtures():
+    d = os.path.join(GOLDEN_DIR, "variant")
+    return sorted(os.path.join(d, f) for f in os.listdir(d) if f.endswith(".txt"))
 
 
 def all_fixtures():
