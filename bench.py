@@ -38,7 +38,17 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 KERNEL_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "kernels.cuh")
 PROFILE_DIR = os.path.join(ROOT, "profiles")
 # rollout kernel launched for each av_rollout_path value
-KERNEL_NAMES = {1: "rollout_kernel", 2: "rollout_fast_kernel", 3: "rollout_env_warp_kernel"}
+KERNEL_NAMES = {1: "rollout_kernel", 2: "rollout_fast_kernel", 3: "rollout_env_warp_kernel",
+                4: "rollout_variant_kernel"}
+VARIANT_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_variant.cu")
+
+
+def bench_variant(wl) -> dict:
+    """Variant semantics of the --variant runs: every rule applied at most once
+    per step, chosen by random index values; rule r inhibits rule r + 1."""
+    R = wl.n_rules
+    return dict(random_keys=1, key_seed=12345, limit=[1] * R,
+                inhibit=[1 << ((r + 1) % R) for r in range(R)])
 SM_COUNT_GB300 = 152
 # 32-bit integer instructions issued per SM per clock: 4 schedulers x 32 lanes.
 # The committed probe (--int-probe) reaches 113-114 of them for IADD3, SHF and
@@ -214,9 +224,11 @@ def profile_traffic(kernel: str, wl, src: str = KERNEL_SRC) -> float | None:
     return float(t.group(1)) if cur.startswith(m.group(1)) else None
 
 
-def cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0) -> dict:
-    """The oracle as it stands, all host cores, on a bounded sample of envs."""
+def cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0, variant=None) -> dict:
+    """The oracle as it stands, all host cores, on a bounded sample of envs
+    (variant: the variant semantics of the run, as keyword arguments)."""
     import oracle
+    ov = oracle.make_variant(**variant) if variant else None
     threads = os.cpu_count() or 1
     s = wk.seeds(seed)
     n = max(threads, 8)
@@ -226,7 +238,7 @@ def cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0) -> dict:
         g = oracle.reset(cfg, cum, s["reset"], ids)
         t0 = time.perf_counter()
         oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), steps, s["actions"], env_ids=ids,
-                       threads=threads)
+                       threads=threads, variant=ov)
         dt = time.perf_counter() - t0
         if dt > budget_s / 4 or n >= wl.batch:
             break
@@ -249,15 +261,16 @@ def run_reference(args, wl):
     s = wk.seeds(args.seed)
     n = max(threads, 16)
     ids = np.arange(n)
+    ov = oracle.make_variant(**bench_variant(wl)) if args.variant else None
     g = oracle.reset(cfg, cum, s["reset"], ids)
     for _ in range(args.warmup):
         oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), 50, s["actions"], env_ids=ids,
-                       threads=threads)
+                       threads=threads, variant=ov)
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
         oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), wl.steps, s["actions"],
-                       env_ids=ids, threads=threads)
+                       env_ids=ids, threads=threads, variant=ov)
         times.append(time.perf_counter() - t0)
     mean = sum(times) / len(times)
     value = n * wl.steps / mean
@@ -265,7 +278,9 @@ def run_reference(args, wl):
         "impl": "reference", "metric": "env-steps/s", "value": value, "unit": "env-steps/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
-        "data": "synthetic", "config": config_dict(wl, sample=n),
+        "data": "synthetic",
+        "config": dict(config_dict(wl, sample=n), **({"workload": VariantName(wl).name,
+                                                       "variant": bench_variant(wl)} if args.variant else {})),
         "cpu_baseline": {"value": value, "unit": "env-steps/s", "cores": threads,
                          "kind": "oracle",
                          "sample": f"{n} of {wl.batch} envs x {wl.steps} fused steps per step"},
@@ -308,6 +323,8 @@ def run_ours(args, wl):
     _, rules, cum = wk.make(wl, seed)
     fields = wk.config_fields(wl)
     env = av.Env(fields, rules, cum, device=dev)
+    if args.variant:
+        av.av_set_variant(env.h, **bench_variant(wl))
     s = wk.seeds(seed)
     g0 = env.reset(s["reset"])
     stream = torch.cuda.current_stream(dev)
@@ -384,13 +401,17 @@ def run_ours(args, wl):
         peak_ops = SM_COUNT_GB300 * INT_LANES_PER_SM * sm_max * 1e6 / 1e9  # Gop/s
         ops = algorithmic_ops(wl, rules)
         achieved = ops * wl.batch * wl.steps / (kernel_ms / 1e3) / 1e9
-        kernel = KERNEL_NAMES[av.av_rollout_path(env.h)]
-        traffic = profile_traffic(kernel, wl)
+        path = av.av_rollout_path(env.h)
+        kernel = KERNEL_NAMES[path]
+        traffic = (profile_traffic(kernel, VariantName(wl), VARIANT_SRC) if path == av.AV_PATH_VARIANT
+                   else profile_traffic(kernel, wl))
         line = {
             "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
-            "data": "synthetic", "config": config_dict(wl),
+            "data": "synthetic",
+            "config": dict(config_dict(wl), **({"workload": VariantName(wl).name,
+                                                "variant": bench_variant(wl)} if args.variant else {})),
             "cell_rule_updates_per_s": value * wl.H * wl.W * wl.n_rules * 4,
             "valid_anchor_rule_tests_per_s": value * valid_anchor_rules(wl, rules),
             "e2e": {"value": e2e_value, "unit": "env-steps/s",
@@ -415,7 +436,8 @@ def run_ours(args, wl):
         if world == 1 and not args.no_cpu_baseline:
             import oracle
             cfg = oracle.make_cfg(**fields)
-            line["cpu_baseline"] = cpu_baseline(wl, rules, cum, cfg, seed)
+            line["cpu_baseline"] = cpu_baseline(wl, rules, cum, cfg, seed,
+                                                variant=bench_variant(wl) if args.variant else None)
         print(json.dumps(line))
     env.close()
     if world > 1:
@@ -871,6 +893,13 @@ MUTATE_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_mutate.cu")
 MIX64_OPS = 20  # 32-bit operations of one SplitMix64 finaliser (3 xor-shifts, 2 64-bit multiplies, input xor)
 
 
+class VariantName:
+    """Name of a rollout workload run under the benchmark's variant semantics."""
+
+    def __init__(self, wl):
+        self.name = f"{wl.name}-variant"
+
+
 class MutateName:
     """Name of the mutation workload (for its profile summary)."""
 
@@ -1107,6 +1136,9 @@ def main(argv=None):
     ap.add_argument("--observe", type=int, default=0, metavar="WINDOW",
                     help="time av_observe (player-centred patches of this width) on the"
                          " 16,384-env training shape instead of a rollout")
+    ap.add_argument("--variant", action="store_true",
+                    help="run the rollout under variant semantics (apply once by random index,"
+                         " rule r inhibits rule r + 1)")
     ap.add_argument("--mutate", action="store_true",
                     help="time av_mutate (maps and rule tables) on the 16,384-env training shape")
     args = ap.parse_args(argv)

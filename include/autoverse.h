@@ -186,6 +186,38 @@ int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, in
  * AV_EINVAL for a NULL bits with R > 0. */
 int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream);
 
+#define AV_MAX_LIMIT 255 /* applications per rule per step under av_set_variant */
+
+/* Variant rule semantics (av_set_variant). */
+typedef struct {
+    int32_t random_keys;             /* 0: ordered index channel; 1: random     */
+    int32_t _pad;
+    uint64_t key_seed;               /* random index values: counter-draw seed  */
+    int32_t limit[AV_MAX_RULES];     /* 0: every match of rule r applies; k: the
+                                        k matches with the largest keys          */
+    uint64_t inhibit[AV_MAX_RULES];  /* bit s: a raw match of rule r suppresses
+                                        rule s for that step                     */
+} av_variant;
+
+/* Variant semantics for the handle's av_step and av_rollout (Sec. 2.1,
+ * "Possible extensions": a rule may be applied only once or a fixed number of
+ * times, and/or in a random order, the tiles to rewrite chosen by the maximum
+ * over an additional channel of ordered or random index values; masking lets
+ * certain rules inhibit others).  A match is (rule r, rotation j, anchor cell
+ * q = y0*W + x0) and has the key (q << 2) | j, or with random_keys
+ * ((draw(key_seed, 13, b, t, q) >> 48) << 14) | (q << 2) | j for env b whose
+ * step counter is t before the step (draw as for av_rollout's actions), so a
+ * rule's matches have distinct keys.  Each step: every rule with at least one
+ * match (before limits) suppresses the rules in its inhibit mask; each rule
+ * not suppressed applies (writes, pays) its limit[r] matches with the largest
+ * keys, or all of them when limit[r] is 0; the writes then combine as in the
+ * standard step.  v = NULL, or all limits and masks zero, restores the standard
+ * step.  While variants are set, av_rollout_path reports AV_PATH_VARIANT and
+ * av_expand returns AV_ESTATE.  AV_EINVAL for a limit outside 0..AV_MAX_LIMIT,
+ * random_keys not 0 or 1, or a limit or mask bit naming a rule slot >= n_rules.
+ * Host call; takes effect for work enqueued after it. */
+int av_set_variant(av_handle *h, const av_variant *v);
+
 /* Rates and ranges of the mutation operators (av_mutate). */
 typedef struct {
     uint32_t p_map;         /* map bit flip rate x 2^24 (0..2^24)                       */
@@ -296,13 +328,14 @@ int av_warnings(av_handle *h, uint32_t *bits);
  * AV_PATH_BLOCK (one CTA per environment), AV_PATH_FAST (several warps per
  * environment, boards of at most 512 cells and at most 64 rules) or
  * AV_PATH_WARP (one warp per environment, boards of at most 512 cells and at
- * most 16 rules).  The library picks the last that fits, except that rule sets
+ * most 16 rules), or AV_PATH_VARIANT when variant semantics are set
+ * (av_set_variant).  The library picks the last of the first three that fits, except that rule sets
  * expected to keep matching on most steps (estimated by av_create from the
  * rules' leading present terms and the init_cum densities) take the block
  * kernel.  The environment variable AV_KERNEL_PATH=block|fast|warp, read by
  * av_create, forces one for tests and measurements.  Writes the path to
  * *path; AV_EINVAL for a null argument.  No GPU work. */
-enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3 };
+enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3, AV_PATH_VARIANT = 4 };
 int av_rollout_path(av_handle *h, int32_t *path);
 
 /* Static description of a status code. */

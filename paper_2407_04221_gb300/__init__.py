@@ -24,9 +24,11 @@ AV_PATH_BLOCK, AV_PATH_FAST, AV_PATH_WARP = 1, 2, 3
 RULE_BYTES = 408
 EXPORTS = ("av_create", "av_destroy", "av_reset", "av_set_state", "av_get_state", "av_step",
            "av_rollout", "av_expand", "av_search_init", "av_select", "av_select_static", "av_sync",
-           "av_warnings", "av_rollout_path", "av_observe", "av_rule_obs", "av_mutate", "av_strerror",
+           "av_warnings", "av_rollout_path", "av_observe", "av_rule_obs", "av_mutate", "av_set_variant", "av_strerror",
            "av_last_error")
 AV_MAX_WINDOW = 127
+AV_MAX_LIMIT = 255
+AV_PATH_VARIANT = 4
 AV_SELECT_STATIC_MAX_HASHES = 1 << 21
 
 
@@ -39,6 +41,12 @@ class AvConfig(ctypes.Structure):
                 ("ch_wall", ctypes.c_int32), ("border_wall", ctypes.c_int32),
                 ("cum_per_env", ctypes.c_int32), ("init_cum", ctypes.c_void_p),
                 ("search_capacity", ctypes.c_int32)]
+
+
+class AvVariant(ctypes.Structure):
+    _fields_ = [("random_keys", ctypes.c_int32), ("_pad", ctypes.c_int32),
+                ("key_seed", ctypes.c_uint64), ("limit", ctypes.c_int32 * 64),
+                ("inhibit", ctypes.c_uint64 * 64)]
 
 
 class AvMutation(ctypes.Structure):
@@ -86,6 +94,7 @@ def load() -> ctypes.CDLL:
         "av_observe": [vp, vp, i32, vp, vp, up],
         "av_rule_obs": [vp, vp, vp, up],
         "av_mutate": [i32, i32, i32, i32, i32, ctypes.POINTER(AvMutation), u64, vp, vp, up],
+        "av_set_variant": [vp, ctypes.POINTER(AvVariant)],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -247,6 +256,25 @@ def av_observe(h, grids, window: int, obs, player_yx=None, stream=None):
 def av_rule_obs(h, bits, reward=None, stream=None):
     """Binary form of the rule tables: bits [T, R, 4, 5, 5, C+1] uint8, reward [T, R]."""
     _check(h, "av_rule_obs", load().av_rule_obs(h, _ptr(bits), _ptr(reward), _stream(stream)))
+
+
+def av_set_variant(h, random_keys=0, key_seed=0, limit=None, inhibit=None, clear=False):
+    """Variant semantics for av_step / av_rollout (Sec. 2.1, possible
+    extensions): limit[r] applications per step by largest key (ordered or
+    random index channel), inhibit[r] = mask of rules a match of r suppresses.
+    clear=True restores the standard step."""
+    L = load()
+    if clear:
+        _check(h, "av_set_variant", L.av_set_variant(h, None))
+        return
+    v = AvVariant()
+    v.random_keys = int(random_keys)
+    v.key_seed = int(key_seed) & (2**64 - 1)
+    for r, k in enumerate(limit or []):
+        v.limit[r] = int(k)
+    for r, m in enumerate(inhibit or []):
+        v.inhibit[r] = int(m)
+    _check(h, "av_set_variant", L.av_set_variant(h, ctypes.byref(v)))
 
 
 def av_mutate(batch, H, W, C, n_rules, mutation: dict, seed: int, maps=None, rules=None,

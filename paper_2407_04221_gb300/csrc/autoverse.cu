@@ -44,6 +44,8 @@ struct av_handle {
     int32_t *d_n_visited = nullptr; // [B]
     uint32_t vis_mask = 0;          // slots per env - 1 (a power of two >= 2 x capacity, minus one)
     uint32_t *d_rules = nullptr;    // the packed 408-byte records as given, [n_tables][R] (rule observation)
+    VariantParams variant{};        // variant semantics (av_set_variant)
+    bool variant_on = false;        // some rule is limited or inhibits another
     bool has_cum = false;
     std::string last_error;
 };
@@ -614,6 +616,12 @@ int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, ui
 {
     if (!h || !actions)
         return AV_EINVAL;
+    if (h->variant_on) {
+        launch_rollout_variant(h->cf, h->variant, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur,
+                               h->d_init, h->d_t, 1, 0, actions, obs, reward, done, nullptr, h->d_status,
+                               as_stream(stream));
+        return launch_check(h, "variant step kernel");
+    }
     launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur, h->d_init, h->d_t, 1, 0,
                    actions, obs, reward, done, nullptr, h->d_status, as_stream(stream));
     return launch_check(h, "step kernel");
@@ -626,6 +634,12 @@ int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_tr
         return AV_EINVAL;
     if (n_steps == 0)
         return AV_OK;
+    if (h->variant_on) {
+        launch_rollout_variant(h->cf, h->variant, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur,
+                               h->d_init, h->d_t, n_steps, action_seed, nullptr, obs_traj, rew_traj, done_traj,
+                               rew_sum, h->d_status, as_stream(stream));
+        return launch_check(h, "variant rollout kernel");
+    }
     launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur, h->d_init, h->d_t, n_steps,
                    action_seed, nullptr, obs_traj, rew_traj, done_traj, rew_sum, h->d_status,
                    as_stream(stream));
@@ -642,6 +656,8 @@ int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_par
         return AV_EINVAL;
     if (F == 0)
         return AV_OK;
+    if (h->variant_on)
+        return fail(h, AV_ESTATE, "av_expand: variant semantics are set (av_set_variant); expansion uses the standard step");
     launch_expand(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, parents, F, n_parent, children, rewards,
                   done, hashes, as_stream(stream));
     return launch_check(h, "expand kernel");
@@ -671,6 +687,36 @@ int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream)
         return AV_EINVAL;
     launch_rule_obs((int)n, h->cf.C, h->d_rules, bits, reward, as_stream(stream));
     return launch_check(h, "rule observation kernel");
+}
+
+int av_set_variant(av_handle *h, const av_variant *v)
+{
+    if (!h)
+        return AV_EINVAL;
+    VariantParams p{};
+    bool on = false;
+    if (v) {
+        const int R = h->cf.R;
+        const uint64_t rules = R >= 64 ? ~0ull : ((1ull << R) - 1ull);
+        if (v->random_keys != 0 && v->random_keys != 1)
+            return fail(h, AV_EINVAL, "av_set_variant: random_keys must be 0 or 1");
+        for (int r = 0; r < AV_MAX_RULES; ++r) {
+            if (v->limit[r] < 0 || v->limit[r] > AV_MAX_LIMIT)
+                return fail(h, AV_EINVAL, "av_set_variant: limits must be in 0..AV_MAX_LIMIT");
+            if (r >= R && (v->limit[r] != 0 || v->inhibit[r] != 0))
+                return fail(h, AV_EINVAL, "av_set_variant: limit or inhibit set for a rule slot >= n_rules");
+            if (v->inhibit[r] & ~rules)
+                return fail(h, AV_EINVAL, "av_set_variant: inhibit mask names a rule slot >= n_rules");
+            p.limit[r] = v->limit[r];
+            p.inhibit[r] = v->inhibit[r];
+            on = on || v->limit[r] != 0 || v->inhibit[r] != 0;
+        }
+        p.random_keys = v->random_keys;
+        p.key_seed = v->key_seed;
+    }
+    h->variant = p;
+    h->variant_on = on;
+    return AV_OK;
 }
 
 int av_mutate(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t n_rules, const av_mutation *m,
@@ -832,7 +878,10 @@ int av_rollout_path(av_handle *h, int32_t *path)
 {
     if (!h || !path)
         return AV_EINVAL;
-    *path = use_env_warp_rollout(h->cf) ? AV_PATH_WARP : use_fast_rollout(h->cf) ? AV_PATH_FAST : AV_PATH_BLOCK;
+    *path = h->variant_on              ? AV_PATH_VARIANT
+            : use_env_warp_rollout(h->cf) ? AV_PATH_WARP
+            : use_fast_rollout(h->cf)     ? AV_PATH_FAST
+                                          : AV_PATH_BLOCK;
     return AV_OK;
 }
 

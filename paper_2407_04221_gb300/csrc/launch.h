@@ -72,6 +72,22 @@ void launch_observe(const DevConfig &cf, const void *grids, int window, uint8_t 
 void launch_rule_obs(int n_rules_total, int C, const uint32_t *rules, uint8_t *bits, int32_t *reward,
                      cudaStream_t st);
 
+// Variant rule semantics (k_variant.cu): apply limits chosen by the largest
+// keys of an ordered or random index channel, inhibition masks.
+struct VariantParams {
+    int32_t random_keys;
+    int32_t pad;
+    uint64_t key_seed;
+    int32_t limit[64];     // 0: every match applies
+    uint64_t inhibit[64];  // bit s: a raw match of rule r suppresses rule s
+};
+cudaError_t configure_variant();
+void launch_rollout_variant(const DevConfig &cf, const VariantParams &vp, const uint32_t *arena,
+                            const uint32_t *tab_off, const uint32_t *vm, const uint32_t *masks, void *cur,
+                            const void *init, int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions,
+                            void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
+                            uint32_t *status, cudaStream_t st);
+
 // Mutation operators (k_mutate.cu).
 void launch_mutate(int B, int H, int W, int C, int R, uint32_t p_map, uint32_t map_channels, uint32_t p_rule,
                    uint32_t p_reward, int32_t reward_min, int32_t reward_max, uint64_t mutable_rules, uint64_t seed,
@@ -87,6 +103,7 @@ inline cudaError_t configure_kernels()
     if (e == cudaSuccess) e = configure_expand();
     if (e == cudaSuccess) e = configure_search();
     if (e == cudaSuccess) e = configure_observe();
+    if (e == cudaSuccess) e = configure_variant();
     return e;
 }
 

@@ -61,6 +61,7 @@ def test_host_side_argument_checks(lib):
     assert lib.av_observe(None, None, 5, None, None, 0) == av.AV_EINVAL
     assert lib.av_rule_obs(None, None, None, 0) == av.AV_EINVAL
     assert lib.av_mutate(1, 16, 16, 8, 8, None, 0, None, None, 0) == av.AV_EINVAL
+    assert lib.av_set_variant(None, None) == av.AV_EINVAL
     m = av.AvMutation(p_map=(1 << 24) + 1)
     assert lib.av_mutate(1, 16, 16, 8, 8, ctypes.byref(m), 0, None, None, 0) == av.AV_EINVAL
     m = av.AvMutation(reward_min=2, reward_max=1)
