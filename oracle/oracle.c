@@ -54,7 +54,7 @@
 #include <stdlib.h>
 #include <string.h>
 
-#define OR_MAXSIDE 64
+#define OR_MAXSIDE 256
 #define OR_MAXCELLS (OR_MAXSIDE * OR_MAXSIDE)
 #define OR_MAXPAT 5
 #define OR_RULE_BYTES 408
@@ -567,23 +567,27 @@ static int run_pool(int n, int threads, void *ctx, int (*fn)(void *, int))
 {
     pool p = {n, threads, ctx, fn, 0, 0};
     pthread_mutex_init(&p.mu, NULL);
-    if (threads <= 1 || n <= 1) {
+    if (threads < 1 || n <= 1)
+        threads = 1;
+    if (threads > 256)
+        threads = 256;
+    /* Workers get large stacks: a 256 x 256 board puts several whole-board
+     * arrays on the stack of each step. */
+    pthread_attr_t attr;
+    pthread_attr_init(&attr);
+    pthread_attr_setstacksize(&attr, (size_t)64 << 20);
+    pthread_t tid[256];
+    int started = 0;
+    for (int i = 0; i < threads; i++)
+        if (pthread_create(&tid[i], &attr, pool_worker, &p) == 0)
+            started++;
+        else
+            break;
+    pthread_attr_destroy(&attr);
+    if (started == 0)
         pool_worker(&p);
-    } else {
-        if (threads > 256)
-            threads = 256;
-        pthread_t tid[256];
-        int started = 0;
-        for (int i = 0; i < threads; i++)
-            if (pthread_create(&tid[i], NULL, pool_worker, &p) == 0)
-                started++;
-            else
-                break;
-        if (started == 0)
-            pool_worker(&p);
-        for (int i = 0; i < started; i++)
-            pthread_join(tid[i], NULL);
-    }
+    for (int i = 0; i < started; i++)
+        pthread_join(tid[i], NULL);
     pthread_mutex_destroy(&p.mu);
     return p.err;
 }

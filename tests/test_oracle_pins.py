@@ -192,16 +192,18 @@ def test_bruteforce_all_3x3_boards_against_convolution(rule_seed):
         np.testing.assert_array_equal(done, ((got >> 1) & 1).sum(axis=(1, 2)) == 0)
 
 
-@pytest.mark.parametrize("key", [1, 2, 3])
+@pytest.mark.parametrize("key", [1, 2, 3, 6])
 def test_random_16x16_against_convolution(key):
-    wl = wk.WORKLOADS[key].scaled(batch=6)
+    """Random boards of the workloads' sizes (16 x 16, and 256 x 256)."""
+    n = 6 if key != 6 else 2
+    wl = wk.WORKLOADS[key].scaled(batch=n)
     rules = wk.make_rules(wl.scaled(rules_per_env=0), 40 + key)
-    g = wk.random_grids(5 + key, 6, wl.H, wl.W, wl.C, density=0.35)
+    g = wk.random_grids(5 + key, n, wl.H, wl.W, wl.C, density=0.35)
     g[:, 3, 4] |= 1 << wk.CH_PLAYER
-    fields = dict(wk.config_fields(wl), batch=6, rules_per_env=0, max_steps=0, auto_reset=0)
+    fields = dict(wk.config_fields(wl), batch=n, rules_per_env=0, max_steps=0, auto_reset=0)
     cfg = oracle.make_cfg(**fields)
-    acts = np.arange(6, dtype=np.uint8) % 5
-    got, _, rew, _ = oracle.step(cfg, rules, g, g, np.zeros(6, np.int32), acts)
+    acts = np.arange(n, dtype=np.uint8) % 5 + (key == 6)
+    got, _, rew, _ = oracle.step(cfg, rules, g, g, np.zeros(n, np.int32), acts)
     exp, exp_rew = conv_formulation(g, rules[0], wl.C, wk.CH_PLAYER, acts)
     np.testing.assert_array_equal(got.astype(np.int64), exp)
     np.testing.assert_array_equal(rew.astype(np.int64), exp_rew)
@@ -268,19 +270,20 @@ def test_single_mover_conserves_counts():
 ROT_ACTION = {0: 0, 1: 4, 2: 1, 3: 2, 4: 3}  # action after a CCW quarter turn
 
 
-@pytest.mark.parametrize("key", [2, 3])
+@pytest.mark.parametrize("key", [2, 3, 6])
 def test_rotation_commutes_with_step(key):
-    wl = wk.WORKLOADS[key].scaled(batch=10)
+    wl = wk.WORKLOADS[key].scaled(batch=10 if key != 6 else 2)
     _, rules, cum = wk.make(wl, 21)
     cfg = _cfg(wl)
-    g = oracle.reset(cfg, cum, 121, range(10))
-    g = g | wk.random_grids(8, 10, wl.H, wl.W, wl.C, density=0.08)
+    n = wl.batch
+    g = oracle.reset(cfg, cum, 121, range(n))
+    g = g | wk.random_grids(8, n, wl.H, wl.W, wl.C, density=0.08)
     for a in range(5):
-        acts = np.full(10, a, np.uint8)
-        out, _, rew, _ = oracle.step(cfg, rules, g, g, np.zeros(10), acts)
+        acts = np.full(n, a, np.uint8)
+        out, _, rew, _ = oracle.step(cfg, rules, g, g, np.zeros(n), acts)
         g_rot = np.ascontiguousarray(np.rot90(g, 1, axes=(1, 2)))
-        acts_rot = np.full(10, ROT_ACTION[a], np.uint8)
-        out_rot, _, rew_rot, _ = oracle.step(cfg, rules, g_rot, g_rot, np.zeros(10), acts_rot)
+        acts_rot = np.full(n, ROT_ACTION[a], np.uint8)
+        out_rot, _, rew_rot, _ = oracle.step(cfg, rules, g_rot, g_rot, np.zeros(n), acts_rot)
         np.testing.assert_array_equal(out_rot, np.rot90(out, 1, axes=(1, 2)))
         np.testing.assert_array_equal(rew_rot, rew)
 

@@ -153,6 +153,9 @@ WORKLOADS = {
                 0.1, 0.1, -3, 3, init="maze", frontier=256, iterations=50, base_game=True),
     5: Workload(5, "grid64-b4096-c16-r24", 4096, 64, 64, 16, 24, ((3, 3), (5, 5)), 0.1,
                 0.1, 0.1, 0.1, -5, 5, steps=500),
+    # boards larger than one CTA's shared memory (the band-streamed rollout)
+    6: Workload(6, "grid256-b256-c16-r24", 256, 256, 256, 16, 24, ((3, 3), (5, 5)), 0.1,
+                0.1, 0.1, 0.1, -5, 5, steps=50),
 }
 
 
