@@ -39,8 +39,9 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "kernels.cuh")
 PROFILE_DIR = os.path.join(ROOT, "profiles")
 # rollout kernel launched for each av_rollout_path value
 KERNEL_NAMES = {1: "rollout_kernel", 2: "rollout_fast_kernel", 3: "rollout_env_warp_kernel",
-                4: "rollout_variant_kernel"}
+                4: "rollout_variant_kernel", 5: "rollout_band_kernel"}
 VARIANT_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_variant.cu")
+BAND_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_band.cu")
 
 
 def bench_variant(wl) -> dict:
@@ -404,6 +405,7 @@ def run_ours(args, wl):
         path = av.av_rollout_path(env.h)
         kernel = KERNEL_NAMES[path]
         traffic = (profile_traffic(kernel, VariantName(wl), VARIANT_SRC) if path == av.AV_PATH_VARIANT
+                   else profile_traffic(kernel, wl, BAND_SRC) if path == av.AV_PATH_BAND
                    else profile_traffic(kernel, wl))
         line = {
             "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
@@ -1125,7 +1127,7 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--config", type=int, default=2, choices=(2, 3, 4, 5))
+    ap.add_argument("--config", type=int, default=2, choices=(2, 3, 4, 5, 6))
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,

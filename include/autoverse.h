@@ -62,18 +62,26 @@ enum {
 /* warning bits reported by av_warnings() */
 enum { AV_WARN_ACTION = 1 /* an action value >= 5 was treated as no-op */ };
 
-#define AV_MAX_SIDE 64   /* H, W <= 64                                   */
+#define AV_MAX_SIDE 256  /* H, W <= 256                                  */
+#define AV_MAX_SMEM_CELLS 4096 /* boards of at most this many cells (64 x 64) stay in one
+                                  CTA's shared memory and support every call; larger
+                                  boards support av_reset, av_set_state, av_get_state,
+                                  av_step, av_rollout (streamed in bands of rows,
+                                  AV_PATH_BAND), av_mutate and av_rule_obs, and return
+                                  AV_EINVAL from av_expand, av_search_init, av_select,
+                                  av_select_static, av_observe and av_set_variant with
+                                  variants */
 #define AV_MAX_C 16      /* C <= 16 tile channels (+1 force channel)     */
 #define AV_MAX_PATTERN 5 /* rule patterns up to 5 x 5                    */
 #define AV_MAX_RULES 64  /* rules per table                              */
-#define AV_MAX_WINDOW 127 /* observation patches up to 127 x 127 (2 * AV_MAX_SIDE - 1) */
+#define AV_MAX_WINDOW 127 /* observation patches up to 127 x 127 (2 * 64 - 1) */
 
 typedef struct av_handle av_handle; /* opaque; owns all env state on the device */
 
 /* Configuration, copied by av_create. */
 typedef struct {
     int32_t batch;         /* B >= 1 environments                                   */
-    int32_t H, W;          /* 1..AV_MAX_SIDE                                        */
+    int32_t H, W;          /* 1..AV_MAX_SIDE (see AV_MAX_SMEM_CELLS)                */
     int32_t C;             /* 1..AV_MAX_C tile channels; force is channel C         */
     int32_t n_rules;       /* R rules per table, 0..AV_MAX_RULES                    */
     int32_t rules_per_env; /* 1: rules[B][R]; 0: one table rules[R] for all envs    */
@@ -328,14 +336,16 @@ int av_warnings(av_handle *h, uint32_t *bits);
  * AV_PATH_BLOCK (one CTA per environment), AV_PATH_FAST (several warps per
  * environment, boards of at most 512 cells and at most 64 rules) or
  * AV_PATH_WARP (one warp per environment, boards of at most 512 cells and at
- * most 16 rules), or AV_PATH_VARIANT when variant semantics are set
- * (av_set_variant).  The library picks the last of the first three that fits, except that rule sets
+ * most 16 rules), AV_PATH_VARIANT when variant semantics are set
+ * (av_set_variant), or AV_PATH_BAND for boards of more than AV_MAX_SMEM_CELLS
+ * cells (one CTA per environment streams the board through shared memory in
+ * bands of rows).  The library picks the last of the first three that fits, except that rule sets
  * expected to keep matching on most steps (estimated by av_create from the
  * rules' leading present terms and the init_cum densities) take the block
  * kernel.  The environment variable AV_KERNEL_PATH=block|fast|warp, read by
  * av_create, forces one for tests and measurements.  Writes the path to
  * *path; AV_EINVAL for a null argument.  No GPU work. */
-enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3, AV_PATH_VARIANT = 4 };
+enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3, AV_PATH_VARIANT = 4, AV_PATH_BAND = 5 };
 int av_rollout_path(av_handle *h, int32_t *path);
 
 /* Static description of a status code. */

@@ -29,6 +29,8 @@ EXPORTS = ("av_create", "av_destroy", "av_reset", "av_set_state", "av_get_state"
 AV_MAX_WINDOW = 127
 AV_MAX_LIMIT = 255
 AV_PATH_VARIANT = 4
+AV_PATH_BAND = 5
+AV_MAX_SMEM_CELLS = 4096
 AV_SELECT_STATIC_MAX_HASHES = 1 << 21
 
 

@@ -44,6 +44,10 @@ struct av_handle {
     int32_t *d_n_visited = nullptr; // [B]
     uint32_t vis_mask = 0;          // slots per env - 1 (a power of two >= 2 x capacity, minus one)
     uint32_t *d_rules = nullptr;    // the packed 408-byte records as given, [n_tables][R] (rule observation)
+    bool large = false;             // more than AV_MAX_SMEM_CELLS cells: the band rollout
+    int band_rows = 0, band_nw = 0; // rows of anchors per band, plane words per band window
+    uint32_t *d_bplanes = nullptr;  // [B][C+1][NW] the boards as bit-planes during a band rollout
+    uint32_t *d_bset = nullptr, *d_bclr = nullptr, *d_bbase = nullptr;  // [B][C][NW]
     VariantParams variant{};        // variant semantics (av_set_variant)
     bool variant_on = false;        // some rule is limited or inhibits another
     bool has_cum = false;
@@ -97,7 +101,7 @@ int check_config(const av_config *c, std::string &why)
 {
     auto bad = [&](const char *m) { why = m; return AV_EINVAL; };
     if (c->batch < 1) return bad("batch must be >= 1");
-    if (c->H < 1 || c->H > AV_MAX_SIDE || c->W < 1 || c->W > AV_MAX_SIDE) return bad("H, W must be in 1..64");
+    if (c->H < 1 || c->H > AV_MAX_SIDE || c->W < 1 || c->W > AV_MAX_SIDE) return bad("H, W must be in 1..256");
     if (c->C < 1 || c->C > AV_MAX_C) return bad("C must be in 1..16");
     if (c->n_rules < 0 || c->n_rules > AV_MAX_RULES) return bad("n_rules must be in 0..64");
     if (c->rules_per_env != 0 && c->rules_per_env != 1) return bad("rules_per_env must be 0 or 1");
@@ -376,6 +380,10 @@ void free_all(av_handle *h)
     cudaFree(h->d_vzero);
     cudaFree(h->d_n_visited);
     cudaFree(h->d_rules);
+    cudaFree(h->d_bplanes);
+    cudaFree(h->d_bset);
+    cudaFree(h->d_bclr);
+    cudaFree(h->d_bbase);
 }
 
 cudaStream_t as_stream(uintptr_t s) { return reinterpret_cast<cudaStream_t>(s); }
@@ -436,6 +444,12 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     cf.NW = (cf.HW + 31) / 32;
     cf.NA = anchor_slots(cf.NW);
     cf.NWP = 8 * cf.NA + kPlanePad;
+    if (cf.HW > AV_MAX_SMEM_CELLS) {
+        // bands of rows through shared memory: the rule tables address the
+        // band window's planes, the lanes cover its words
+        h->large = true;
+        band_geometry(cf.H, cf.W, &h->band_rows, &h->band_nw, &cf.NA, &cf.NWP);
+    }
     cf.R = cfg->n_rules;
     cf.rules_per_env = cfg->rules_per_env;
     cf.max_steps = cfg->max_steps;
@@ -523,6 +537,15 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
             return rc ? rc : AV_ECUDA;
         }
         h->has_cum = true;
+    }
+    if (h->large) {
+        const size_t words = B * (size_t)cf.NW;
+        if ((rc = dalloc(h, &h->d_bplanes, words * (cf.C + 1))) || (rc = dalloc(h, &h->d_bset, words * cf.C)) ||
+            (rc = dalloc(h, &h->d_bclr, words * cf.C)) || (rc = dalloc(h, &h->d_bbase, words * cf.C))) {
+            free_all(h);
+            delete h;
+            return rc;
+        }
     }
     if (cfg->search_capacity > 0) {
         size_t slots = 64;
@@ -616,6 +639,12 @@ int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, ui
 {
     if (!h || !actions)
         return AV_EINVAL;
+    if (h->large) {
+        launch_rollout_band(h->cf, h->band_rows, h->band_nw, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks,
+                            h->d_cur, h->d_init, h->d_t, 1, 0, actions, obs, reward, done, nullptr, h->d_status,
+                            h->d_bplanes, h->d_bset, h->d_bclr, h->d_bbase, as_stream(stream));
+        return launch_check(h, "band step kernel");
+    }
     if (h->variant_on) {
         launch_rollout_variant(h->cf, h->variant, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur,
                                h->d_init, h->d_t, 1, 0, actions, obs, reward, done, nullptr, h->d_status,
@@ -634,6 +663,13 @@ int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_tr
         return AV_EINVAL;
     if (n_steps == 0)
         return AV_OK;
+    if (h->large) {
+        launch_rollout_band(h->cf, h->band_rows, h->band_nw, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks,
+                            h->d_cur, h->d_init, h->d_t, n_steps, action_seed, nullptr, obs_traj, rew_traj,
+                            done_traj, rew_sum, h->d_status, h->d_bplanes, h->d_bset, h->d_bclr, h->d_bbase,
+                            as_stream(stream));
+        return launch_check(h, "band rollout kernel");
+    }
     if (h->variant_on) {
         launch_rollout_variant(h->cf, h->variant, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur,
                                h->d_init, h->d_t, n_steps, action_seed, nullptr, obs_traj, rew_traj, done_traj,
@@ -654,6 +690,8 @@ int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_par
         return AV_EINVAL;
     if ((size_t)h->cf.B * (size_t)F > 0x7fffffffu)
         return AV_EINVAL;
+    if (h->large)
+        return fail(h, AV_EINVAL, "av_expand: boards over AV_MAX_SMEM_CELLS cells are not supported");
     if (F == 0)
         return AV_OK;
     if (h->variant_on)
@@ -672,6 +710,8 @@ int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, in
         return fail(h, AV_EINVAL, "av_observe: window must be in 1..AV_MAX_WINDOW");
     if (h->cf.ch_player < 0)
         return fail(h, AV_ESTATE, "av_observe: the configuration has no player channel");
+    if (h->large)
+        return fail(h, AV_EINVAL, "av_observe: boards over AV_MAX_SMEM_CELLS cells are not supported");
     if ((size_t)h->cf.B > 0x7fffffffu)
         return AV_EINVAL;
     launch_observe(h->cf, grids ? grids : h->d_cur, window, obs, player_yx, as_stream(stream));
@@ -713,6 +753,8 @@ int av_set_variant(av_handle *h, const av_variant *v)
         }
         p.random_keys = v->random_keys;
         p.key_seed = v->key_seed;
+        if (on && h->large)
+            return fail(h, AV_EINVAL, "av_set_variant: boards over AV_MAX_SMEM_CELLS cells are not supported");
     }
     h->variant = p;
     h->variant_on = on;
@@ -742,6 +784,8 @@ int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t
         return AV_EINVAL;
     if (h->host_cfg.search_capacity < 1)
         return fail(h, AV_ESTATE, "av_search_init: search_capacity is 0");
+    if (h->large)
+        return fail(h, AV_EINVAL, "av_search_init: boards over AV_MAX_SMEM_CELLS cells are not supported");
     const cudaStream_t st = as_stream(stream);
     AV_CUDA(h, cudaMemsetAsync(h->d_vtab, 0, (size_t)h->cf.B * (h->vis_mask + 1) * sizeof(uint64_t), st));
     AV_CUDA(h, cudaMemsetAsync(h->d_vzero, 0, (size_t)h->cf.B * sizeof(uint32_t), st));
@@ -760,6 +804,8 @@ int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *p
         return AV_EINVAL;
     if (h->host_cfg.search_capacity < 1)
         return fail(h, AV_ESTATE, "av_select: search_capacity is 0");
+    if (h->large)
+        return fail(h, AV_EINVAL, "av_select: boards over AV_MAX_SMEM_CELLS cells are not supported");
     if (F < 1 || 5 * F > kMaxCand || k < 1 || k > 5 * F)
         return fail(h, AV_EINVAL, "av_select: need 1 <= F, 5*F <= 4096, 1 <= k <= 5*F");
     if (!n_parent || !parent_cum || !parent_live || !cand_grids || !cand_reward || !cand_done ||
@@ -819,7 +865,8 @@ int av_select_static(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t F,
                      uint64_t *next_hash, uint8_t *next_live, int32_t *n_next, uint64_t *visited,
                      int32_t *n_visited, int32_t capacity, uint32_t *status, uintptr_t stream)
 {
-    if (batch < 1 || H < 1 || H > AV_MAX_SIDE || W < 1 || W > AV_MAX_SIDE || C < 1 || C > AV_MAX_C)
+    if (batch < 1 || H < 1 || H > AV_MAX_SIDE || W < 1 || W > AV_MAX_SIDE || C < 1 || C > AV_MAX_C ||
+        H * W > AV_MAX_SMEM_CELLS)
         return AV_EINVAL;
     if (F < 1 || 5 * F > kMaxCand || k < 1 || k > 5 * F || capacity < 1)
         return AV_EINVAL;
@@ -878,7 +925,8 @@ int av_rollout_path(av_handle *h, int32_t *path)
 {
     if (!h || !path)
         return AV_EINVAL;
-    *path = h->variant_on              ? AV_PATH_VARIANT
+    *path = h->large                   ? AV_PATH_BAND
+            : h->variant_on            ? AV_PATH_VARIANT
             : use_env_warp_rollout(h->cf) ? AV_PATH_WARP
             : use_fast_rollout(h->cf)     ? AV_PATH_FAST
                                           : AV_PATH_BLOCK;

@@ -88,6 +88,16 @@ void launch_rollout_variant(const DevConfig &cf, const VariantParams &vp, const 
                             void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
                             uint32_t *status, cudaStream_t st);
 
+// Boards larger than one CTA's shared memory (k_band.cu): the step streamed
+// through shared memory in bands of rows.
+cudaError_t configure_band();
+void band_geometry(int H, int W, int *band_rows, int *band_nw, int *na, int *nwp);
+void launch_rollout_band(const DevConfig &cf, int band_rows, int band_nw, const uint32_t *arena,
+                         const uint32_t *tab_off, const uint32_t *vm, const uint32_t *masks, void *cur,
+                         const void *init, int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions,
+                         void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                         uint32_t *planes, uint32_t *set, uint32_t *clr, uint32_t *base, cudaStream_t st);
+
 // Mutation operators (k_mutate.cu).
 void launch_mutate(int B, int H, int W, int C, int R, uint32_t p_map, uint32_t map_channels, uint32_t p_rule,
                    uint32_t p_reward, int32_t reward_min, int32_t reward_max, uint64_t mutable_rules, uint64_t seed,
@@ -104,6 +114,7 @@ inline cudaError_t configure_kernels()
     if (e == cudaSuccess) e = configure_search();
     if (e == cudaSuccess) e = configure_observe();
     if (e == cudaSuccess) e = configure_variant();
+    if (e == cudaSuccess) e = configure_band();
     return e;
 }
 
