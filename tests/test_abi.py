@@ -67,11 +67,11 @@ def test_host_side_argument_checks(lib):
     m = av.AvMutation(reward_min=2, reward_max=1)
     assert lib.av_mutate(1, 16, 16, 8, 8, ctypes.byref(m), 0, None, None, 0) == av.AV_EINVAL
     m = av.AvMutation()
-    assert lib.av_mutate(1, 65, 16, 8, 8, ctypes.byref(m), 0, None, None, 0) == av.AV_EINVAL
+    assert lib.av_mutate(1, 257, 16, 8, 8, ctypes.byref(m), 0, None, None, 0) == av.AV_EINVAL
     assert av.av_strerror(av.AV_EINVAL) == "invalid argument"
     base = dict(batch=1, H=16, W=16, C=4, n_rules=0, rules_per_env=0, max_steps=0, auto_reset=0,
                 ch_player=2, ch_goal=3, ch_empty=0, ch_wall=1, border_wall=1, cum_per_env=0)
-    bad = [dict(batch=0), dict(H=65), dict(W=0), dict(C=17), dict(C=0), dict(n_rules=65),
+    bad = [dict(batch=0), dict(H=257), dict(W=0), dict(C=17), dict(C=0), dict(n_rules=65),
            dict(ch_goal=4), dict(ch_player=-2), dict(rules_per_env=2), dict(max_steps=-1)]
     for b in bad:
         with pytest.raises(av.AvError) as ei:
