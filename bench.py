@@ -324,6 +324,7 @@ def run_ours(args, wl):
     _, rules, cum = wk.make(wl, seed)
     fields = wk.config_fields(wl)
     env = av.Env(fields, rules, cum, device=dev)
+    std_path = av.av_rollout_path(env.h)
     if args.variant:
         av.av_set_variant(env.h, **bench_variant(wl))
     s = wk.seeds(seed)
@@ -404,6 +405,8 @@ def run_ours(args, wl):
         achieved = ops * wl.batch * wl.steps / (kernel_ms / 1e3) / 1e9
         path = av.av_rollout_path(env.h)
         kernel = KERNEL_NAMES[path]
+        if path == av.AV_PATH_VARIANT and std_path == av.AV_PATH_WARP:
+            kernel = "rollout_variant_warp_kernel"  # variants on the one-warp layout
         traffic = (profile_traffic(kernel, VariantName(wl), VARIANT_SRC) if path == av.AV_PATH_VARIANT
                    else profile_traffic(kernel, wl, BAND_SRC) if path == av.AV_PATH_BAND
                    else profile_traffic(kernel, wl))

@@ -53,8 +53,15 @@ def test_variant_fixture(path):
 
 @pytest.mark.parametrize("key", [1, 2, 3, 4, 5])
 @pytest.mark.parametrize("random_keys", [0, 1])
-def test_rollout_every_shape(key, random_keys):
+@pytest.mark.parametrize("kernel", ["default", "warp", "block"])
+def test_rollout_every_shape(key, random_keys, kernel, monkeypatch):
+    """Both variant kernels (one warp per environment, one CTA per
+    environment) on every shape the first supports."""
     import paper_2407_04221_gb300 as av
+    if kernel != "default":
+        if key == 5 and kernel == "warp":
+            pytest.skip("64 x 64 boards take the CTA-per-environment kernel")
+        monkeypatch.setenv("AV_KERNEL_PATH", kernel)
     n = 24 if key != 5 else 8
     steps = 40 if key != 5 else 12
     wl = wk.WORKLOADS[key].scaled(batch=n)
