@@ -37,7 +37,38 @@ CASES = {
     "17x256-c16-dense": (DENSE, dict(batch=3, H=17, W=256)),
     "96x96-c16-dense": (DENSE, dict(batch=3, H=96, W=96)),
     "200x33-c8": (wk.WORKLOADS[2], dict(batch=4, H=200, W=33)),
+    "256x256-c16-r64-dense": (DENSE, dict(batch=2, H=256, W=256, n_rules=64)),  # every limit at once
 }
+
+
+def _one_channel_rules():
+    """Two hand-made rules on one tile channel: a lit cell goes dark, and a
+    dark cell left of a lit one lights up (both every step, in parallel)."""
+    r = wk.empty_rules(1, 2)
+    r[0, 0]["h"], r[0, 0]["w"], r[0, 0]["reward"] = 1, 1, 1
+    r[0, 0]["present"][0], r[0, 0]["clear"][0] = 1, 1
+    r[0, 1]["h"], r[0, 1]["w"], r[0, 1]["reward"] = 1, 2, -1
+    r[0, 1]["absent"][0], r[0, 1]["present"][1], r[0, 1]["set"][0] = 1, 1, 1
+    return r
+
+
+def test_one_channel_256x256():
+    """C = 1 (no player, no goal): the smallest cell and the largest board."""
+    import paper_2407_04221_gb300 as av
+    fields = dict(batch=2, H=256, W=256, C=1, n_rules=2, rules_per_env=0, max_steps=0, auto_reset=0,
+                  ch_player=-1, ch_goal=-1, ch_empty=-1, ch_wall=-1, border_wall=0, cum_per_env=0)
+    rules = _one_channel_rules()
+    g0 = wk.random_grids(4, 2, 256, 256, 1, density=0.3)
+    env = av.Env(fields, rules)
+    assert av.av_rollout_path(env.h) == av.AV_PATH_BAND
+    env.set_state(to_dev(g0), set_as_init=True)
+    res = env.rollout(10, 5, trajectory=True)
+    cfg = oracle.make_cfg(**fields)
+    ref = oracle.rollout(cfg, rules, g0, g0, np.zeros(2, np.int32), 10, 5, trajectory=True)
+    assert (ref["obs"][0] != g0).any()
+    np.testing.assert_array_equal(to_np(res["obs"]), ref["obs"])
+    np.testing.assert_array_equal(to_np(res["rew"]), ref["rew"])
+    env.close()
 
 
 @pytest.mark.parametrize("case", list(CASES))

@@ -162,6 +162,7 @@ def test_step_random_actions(key):
     (2, 64, 9, ((1, 5), (2, 2)), 3),            # short and wide, 2-byte cells
     (33, 33, 8, ((5, 5), (3, 1)), 5),           # rows straddle 32-bit words
     (64, 64, 4, ((5, 5),), 1),
+    (64, 64, 16, ((5, 5), (3, 3), (1, 2)), 64),  # the largest board, channels and rules in one CTA
 ])
 def test_edge_shapes(H, W, C, shapes, R):
     wl = wk.Workload(0, "edge", 3, H, W, C, R, shapes, 0.12, 0.08, 0.2, 0.2, -2, 2,
@@ -247,6 +248,7 @@ def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
     (16, 16, 5, ((1, 1), (1, 2)), 40),  # many rules: several per warp
     (16, 16, 5, ((1, 1), (1, 2)), 16),  # the most rules one warp per environment holds
     (12, 16, 4, ((2, 2), (1, 3)), 11),
+    (16, 16, 8, ((3, 3), (1, 2), (5, 5)), 64),  # the most rules a table holds
 ])
 def test_both_kernel_paths_edges(monkeypatch, path, H, W, C, shapes, R):
     import paper_2407_04221_gb300 as av
