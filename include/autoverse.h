@@ -67,9 +67,9 @@ enum { AV_WARN_ACTION = 1 /* an action value >= 5 was treated as no-op */ };
                                   CTA's shared memory and support every call; larger
                                   boards support av_reset, av_set_state, av_get_state,
                                   av_step, av_rollout (streamed in bands of rows,
-                                  AV_PATH_BAND), av_mutate and av_rule_obs, and return
-                                  AV_EINVAL from av_expand, av_search_init, av_select,
-                                  av_select_static, av_observe and av_set_variant with
+                                  AV_PATH_BAND), av_observe, av_mutate and av_rule_obs,
+                                  and return AV_EINVAL from av_expand, av_search_init,
+                                  av_select, av_select_static and av_set_variant with
                                   variants */
 #define AV_MAX_C 16      /* C <= 16 tile channels (+1 force channel)     */
 #define AV_MAX_PATTERN 5 /* rule patterns up to 5 x 5                    */

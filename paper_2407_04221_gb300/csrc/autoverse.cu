@@ -710,8 +710,6 @@ int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, in
         return fail(h, AV_EINVAL, "av_observe: window must be in 1..AV_MAX_WINDOW");
     if (h->cf.ch_player < 0)
         return fail(h, AV_ESTATE, "av_observe: the configuration has no player channel");
-    if (h->large)
-        return fail(h, AV_EINVAL, "av_observe: boards over AV_MAX_SMEM_CELLS cells are not supported");
     if ((size_t)h->cf.B > 0x7fffffffu)
         return AV_EINVAL;
     launch_observe(h->cf, grids ? grids : h->d_cur, window, obs, player_yx, as_stream(stream));

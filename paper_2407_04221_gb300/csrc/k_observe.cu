@@ -7,7 +7,8 @@
 // environments (one environment per group for large patches, up to eight for
 // small ones; their boards and patches are contiguous).  A group's boards are
 // fetched into shared memory with cp.async while the previous group's patches
-// are built; each environment's player is its first row-major cell with the
+// are built (boards over 8 KB, up to 256 x 256, are read from global memory
+// instead); each environment's player is its first row-major cell with the
 // player bit (a warp reduction, then an atomicMin).  The patches -- [window]
 // [window][C] bytes each, channels last -- are built in a staging slab that is
 // zero-filled with 16-byte stores, after which only the set tile bits of the
@@ -120,19 +121,20 @@ __global__ void __launch_bounds__(kObsThreads)
     auto group_size = [&](int grp) { return min(E, B - grp * E); };
     if (tid < E)
         s_first[0][tid] = HW;
-    fetch_board(board_at(0), grids + (size_t)g * E * HW, group_size(g) * HW, vec16);
+    if (board_region)  // else boards are read from global memory where they lie
+        fetch_board(board_at(0), grids + (size_t)g * E * HW, group_size(g) * HW, vec16);
     uint32_t unit = 0;  // slabs issued so far; slab buffer = unit & 1
     for (int it = 0; g < n_groups; ++it, g += gridDim.x) {
         const int pb = it & 1;
         const int ne = group_size(g);
-        const CellT *board = board_at(pb);
+        const CellT *board = board_region ? board_at(pb) : grids + (size_t)g * E * HW;
         uint8_t *out = obs + (size_t)g * E * patch_bytes;
         if (tid == 0)
             bulk_wait_read<1>();  // slab_at(unit) has been read by its last store
         cp_async_wait_all();
         __syncthreads();  // the group's boards in shared memory; s_first[pb] reset; slab free
         const int gn = g + gridDim.x;
-        if (gn < n_groups)
+        if (board_region && gn < n_groups)
             fetch_board(board_at(pb ^ 1), grids + (size_t)gn * E * HW, group_size(gn) * HW, vec16);
         // Each environment's player: its first row-major cell holding the
         // player bit.  A thread's first hit is its minimum; a warp reduces its
@@ -266,6 +268,10 @@ struct ObserveLayout {
 // every SM has work.
 constexpr size_t kObsGroupBytes = 20480;
 constexpr size_t kObsGroupBoardBytes = 16384;
+// Boards above this size (the band-streamed ones, over 4096 two-byte cells)
+// are not staged: the player search and the window's cells read them from
+// global memory.
+constexpr size_t kObsStageBoardMax = 8192;
 
 ObserveLayout observe_layout(const DevConfig &cf, int window, int sm_count)
 {
@@ -282,7 +288,7 @@ ObserveLayout observe_layout(const DevConfig &cf, int window, int sm_count)
     }
     L.E = (int)E;
     L.rows = E == 1 ? observe_rows_per_slab(window, cf.C) : window;
-    L.board_region = (int)align16(E * board);
+    L.board_region = board > kObsStageBoardMax ? 0 : (int)align16(E * board);
     L.buf_region = (int)align16((E == 1 ? (size_t)L.rows * window * cf.C : E * patch) + 16);
     L.smem = 2 * (size_t)L.board_region + 2 * (size_t)L.buf_region;
     return L;

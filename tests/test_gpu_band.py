@@ -150,7 +150,7 @@ def test_unsupported_calls_on_large_boards():
     wl = wk.WORKLOADS[2].scaled(batch=2, H=65, W=65)
     env, cfg, rules, cum = make(wl, 0, search_capacity=16)
     parents = env.boards(2, 1)
-    for call in (lambda: env.expand(parents), lambda: env.observe(5),
+    for call in (lambda: env.expand(parents),
                  lambda: av.av_search_init(env.h, env.boards(2),
                                            torch.zeros(2, dtype=torch.int64, device="cuda"),
                                            torch.zeros(2, dtype=torch.uint8, device="cuda")),
@@ -158,4 +158,28 @@ def test_unsupported_calls_on_large_boards():
         with pytest.raises(av.AvError) as ei:
             call()
         assert ei.value.status == av.AV_EINVAL
+    env.close()
+
+
+@pytest.mark.parametrize("H,W,C,window", [(256, 256, 16, 31), (256, 256, 10, 127), (100, 70, 8, 20),
+                                          (65, 65, 3, 5)])
+def test_observation_of_large_boards(H, W, C, window):
+    """Boards too large to stage in shared memory are observed from global
+    memory: players anywhere, none, or several."""
+    import paper_2407_04221_gb300 as av
+    rng = np.random.default_rng(H + W + C)
+    B = 5
+    boards = rng.integers(0, 1 << C, size=(B, H, W)).astype(oracle.cell_dtype(C))
+    boards &= ~np.array(1 << 2, boards.dtype)
+    for b in range(B):
+        for _ in range(b % 3):
+            boards[b, rng.integers(H), rng.integers(W)] |= 1 << 2
+    fields = dict(batch=B, H=H, W=W, C=C, n_rules=0, rules_per_env=0, max_steps=0, auto_reset=0,
+                  ch_player=2, ch_goal=-1, ch_empty=-1, ch_wall=-1, border_wall=0, cum_per_env=0)
+    env = av.Env(fields, np.zeros(0, np.uint8))
+    env.set_state(to_dev(boards))
+    obs, pyx = env.observe(window)
+    want, want_pyx = oracle.observe(oracle.make_cfg(**fields), boards, window)
+    np.testing.assert_array_equal(to_np(obs), want)
+    np.testing.assert_array_equal(to_np(pyx), want_pyx)
     env.close()
