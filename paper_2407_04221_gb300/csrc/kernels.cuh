@@ -513,16 +513,18 @@ rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t 
         match_all<NA, SM>(cf, tab, S);
         __syncthreads();
         if (warp == 0) {
-            // combine: a bit changes where any match asks for it
+            // combine: a bit changes where any match asks for it (one index over
+            // every channel's words, so small boards keep all lanes busy)
             if (S.flags[0]) {
-                for (int c = 0; c < C; ++c)
-                    for (int w = lane; w < NW; w += 32) {
-                        const int i = c * NW + w;
-                        const uint32_t d = S.planes[c * NWP + w].x, st = S.setp[i], cl = S.clrp[i];
-                        S.setp[i] = 0u;
-                        S.clrp[i] = 0u;
-                        put_word(S.planes, NWP, c, w, (d & ~cl) | (~d & st));
-                    }
+                // (c, w) of index i = c * NW + w, stepped without a division
+                for (int i = lane, c = lane / NW, w = lane - (lane / NW) * NW; i < C * NW; i += 32) {
+                    const uint32_t d = S.planes[c * NWP + w].x, st = S.setp[i], cl = S.clrp[i];
+                    S.setp[i] = 0u;
+                    S.clrp[i] = 0u;
+                    put_word(S.planes, NWP, c, w, (d & ~cl) | (~d & st));
+                    for (w += 32; w >= NW; w -= NW)
+                        ++c;
+                }
                 __syncwarp();
                 if (lane == 0)
                     S.flags[0] = 0;
@@ -535,9 +537,11 @@ rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t 
             t += 1;
             const int done = !goal || (cf.max_steps > 0 && t >= cf.max_steps);
             if (done && cf.auto_reset) {
-                for (int c = 0; c < C; ++c)
-                    for (int w = lane; w < NW; w += 32)
-                        put_word(S.planes, NWP, c, w, S.basep[c * NW + w]);
+                for (int i = lane, c = lane / NW, w = lane - (lane / NW) * NW; i < C * NW; i += 32) {
+                    put_word(S.planes, NWP, c, w, S.basep[i]);
+                    for (w += 32; w >= NW; w -= NW)
+                        ++c;
+                }
                 t = 0;
             }
             int rew = lane < kWarps ? S.red[lane] : 0;
@@ -760,6 +764,53 @@ __device__ __forceinline__ int planes_to_cells(const DevConfig &cf, const uint2 
 // (pass 1, four terms per vote); a rule with anchors left then applies its
 // force terms for all five actions at once (pass 2) and writes each action's
 // outputs into that action's SET / CLEAR planes.
+// A child board from its parent's canonical words: a child differs from its
+// parent only where its SET / CLEAR words flip a bit, so each output word is
+// the parent's (tile bits only), rebuilt by planes_to_cells' formula where the
+// plane word under it has a flipped bit.  `parent` (global, 4-byte aligned,
+// whole words) holds the parent's canonical words.  Writes `out` (shared) and
+// `dst` (global, 4-byte aligned); returns whether any goal tile is left.  One
+// warp; boards of at most 32 plane words.
+template <typename CellT>
+__device__ __forceinline__ int child_cells(const DevConfig &cf, const uint2 *dbl, const uint32_t *setp,
+                                           const uint32_t *clrp, const uint32_t *parent, uint32_t *out, CellT *dst)
+{
+    const int lane = threadIdx.x & 31, HW = cf.HW, NW = cf.NW, NWP = cf.NWP;
+    constexpr int kPer = 4 / (int)sizeof(CellT);  // cells per 32-bit word
+    const int n_words = HW / kPer;
+    uint32_t flip = 0, goal = 0;
+    if (lane < NW) {
+        for (int c = 0; c < cf.C; ++c) {
+            const uint32_t d = dbl[c * NWP + lane].x, st = setp[c * NW + lane], cl = clrp[c * NW + lane];
+            flip |= (d & cl) | (~d & st);
+            if (c == cf.ch_goal)
+                goal = (d & ~cl) | (~d & st);
+        }
+    }
+    const uint32_t changed = __ballot_sync(0xffffffffu, flip != 0u);  // plane words with a flipped bit
+    const int goal_left = cf.ch_goal < 0 || __any_sync(0xffffffffu, goal != 0u);
+    const uint32_t tiles = ((1u << cf.C) - 1u) * (sizeof(CellT) == 1 ? 0x01010101u : 0x00010001u);
+    for (int g = lane; g < n_words; g += 32) {
+        const int p0 = g * kPer, j = p0 >> 5, b = p0 & 31;
+        uint32_t v;
+        if ((changed >> j) & 1u) {
+            v = 0;
+            for (int c = 0; c < cf.C; ++c) {
+                const uint32_t d = dbl[c * NWP + j].x, st = setp[c * NW + j], cl = clrp[c * NW + j];
+                const uint32_t x = ((d & ~cl) | (~d & st)) >> b;
+                const uint32_t spread = sizeof(CellT) == 1 ? ((x & 0xfu) * 0x00204081u) & 0x01010101u
+                                                           : ((x & 0x3u) * 0x00008001u) & 0x00010001u;
+                v |= spread << c;
+            }
+        } else {
+            v = __ldg(parent + g) & tiles;
+        }
+        out[g] = v;
+        reinterpret_cast<uint32_t *>(dst)[g] = v;
+    }
+    return goal_left;
+}
+
 template <typename CellT, int NA, bool SM>
 __device__ __forceinline__ void expand_rules(const DevConfig &cf, const uint32_t *tab, const WarpSmem &S,
                                              int (&rew)[5])
@@ -924,11 +975,19 @@ expand_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint3
         int rew[5] = {0, 0, 0, 0, 0};
         expand_rules<CellT, NA, SM>(cf, tab, S, rew);
         __syncwarp();  // every lane's SET / CLEAR bits
+        // children from the parent's words where the board and both pointers
+        // allow whole-word access, else rebuilt from the planes
+        const CellT *par = parents + (size_t)node * HW;
+        const bool words = (HW * (int)sizeof(CellT)) % 4 == 0 && (reinterpret_cast<uintptr_t>(par) & 3u) == 0 &&
+                           (reinterpret_cast<uintptr_t>(children) & 3u) == 0;
 #pragma unroll
         for (int a = 0; a < 5; ++a) {
-            const int goal_left = planes_to_cells<CellT>(cf, S.planes, S.setp + a * C * NW, S.clrp + a * C * NW,
-                                                         bytes + a * (L.child_bytes / 4),
-                                                         children + ((size_t)node * 5 + a) * HW);
+            CellT *dst = children + ((size_t)node * 5 + a) * HW;
+            const int goal_left =
+                words ? child_cells<CellT>(cf, S.planes, S.setp + a * C * NW, S.clrp + a * C * NW,
+                                           reinterpret_cast<const uint32_t *>(par), bytes + a * (L.child_bytes / 4), dst)
+                      : planes_to_cells<CellT>(cf, S.planes, S.setp + a * C * NW, S.clrp + a * C * NW,
+                                               bytes + a * (L.child_bytes / 4), dst);
             const int r = __reduce_add_sync(0xffffffffu, rew[a]);
             if (lane == 0) {
                 rewards[(size_t)node * 5 + a] = r;
