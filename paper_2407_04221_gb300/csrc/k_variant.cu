@@ -229,14 +229,15 @@ __global__ void __launch_bounds__(kThreads)
         if (warp == 0) {
             // combine: a bit changes where any kept match asks for it
             if (S.flags[0]) {
-                for (int c = 0; c < C; ++c)
-                    for (int w = lane; w < NW; w += 32) {
-                        const int i = c * NW + w;
-                        const uint32_t d = S.planes[c * NWP + w].x, st = S.setp[i], cl = S.clrp[i];
-                        S.setp[i] = 0u;
-                        S.clrp[i] = 0u;
-                        put_word(S.planes, NWP, c, w, (d & ~cl) | (~d & st));
-                    }
+                // one index over every channel's words; (c, w) stepped without a division
+                for (int i = lane, c = lane / NW, w = lane - (lane / NW) * NW; i < C * NW; i += 32) {
+                    const uint32_t d = S.planes[c * NWP + w].x, st = S.setp[i], cl = S.clrp[i];
+                    S.setp[i] = 0u;
+                    S.clrp[i] = 0u;
+                    put_word(S.planes, NWP, c, w, (d & ~cl) | (~d & st));
+                    for (w += 32; w >= NW; w -= NW)
+                        ++c;
+                }
                 __syncwarp();
                 if (lane == 0)
                     S.flags[0] = 0;
@@ -249,9 +250,11 @@ __global__ void __launch_bounds__(kThreads)
             int tn = t + 1;
             const int done = !goal || (cf.max_steps > 0 && tn >= cf.max_steps);
             if (done && cf.auto_reset) {
-                for (int c = 0; c < C; ++c)
-                    for (int w = lane; w < NW; w += 32)
-                        put_word(S.planes, NWP, c, w, S.basep[c * NW + w]);
+                for (int i = lane, c = lane / NW, w = lane - (lane / NW) * NW; i < C * NW; i += 32) {
+                    put_word(S.planes, NWP, c, w, S.basep[i]);
+                    for (w += 32; w >= NW; w -= NW)
+                        ++c;
+                }
                 tn = 0;
             }
             int total = lane < kWarps ? S.red[lane] : 0;
