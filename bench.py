@@ -244,9 +244,19 @@ def cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0, variant=None
         if dt > budget_s / 4 or n >= wl.batch:
             break
         n = min(wl.batch, int(n * max(2.0, budget_s / 4 / max(dt, 1e-3))))
+    # The same oracle on one thread, over about one core's share of the sample.
+    m = max(1, n // threads)
+    ids1 = np.arange(m)
+    g1 = oracle.reset(cfg, cum, s["reset"], ids1)
+    t0 = time.perf_counter()
+    oracle.rollout(cfg, rules, g1, g1, np.zeros(m, np.int32), steps, s["actions"], env_ids=ids1,
+                   threads=1, variant=ov)
+    dt1 = time.perf_counter() - t0
     return {"value": n * steps / dt, "unit": "env-steps/s", "cores": threads, "kind": "oracle",
             "sample": f"{n} of {wl.batch} envs x {steps} fused steps (envs are independent)",
-            "seconds": dt}
+            "seconds": dt,
+            "one_thread": {"value": m * steps / dt1, "cores": 1,
+                           "sample": f"{m} of {wl.batch} envs x {steps} fused steps"}}
 
 
 # ------------------------------------------------------------ reference
@@ -639,9 +649,19 @@ def search_cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0) -> di
             break
         n = min(wl.batch, int(n * max(2.0, budget_s / 4 / max(dt, 1e-3))))
     children = 5 * (n + int(ref["trace_n"][:, :-1].sum()))
+    # The same search on one thread, over about one core's share of the sample.
+    m = max(1, n // threads)
+    ids1 = np.arange(m)
+    roots1 = oracle.reset(cfg, cum, s["reset"], ids1)
+    t0 = time.perf_counter()
+    one = oracle.search(cfg, rules, roots1, wl.iterations, wl.frontier, env_ids=ids1, threads=1)
+    dt1 = time.perf_counter() - t0
+    children1 = 5 * (m + int(one["trace_n"][:, :-1].sum()))
     return {"value": children / dt, "unit": "env-steps/s", "cores": threads, "kind": "oracle",
             "sample": f"{n} of {wl.batch} envs, full search ({wl.iterations} iterations,"
-                      f" frontier {wl.frontier})", "seconds": dt}
+                      f" frontier {wl.frontier})", "seconds": dt,
+            "one_thread": {"value": children1 / dt1, "cores": 1,
+                           "sample": f"{m} of {wl.batch} envs, full search"}}
 
 
 def run_search_reference(args, wl):
