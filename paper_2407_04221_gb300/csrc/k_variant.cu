@@ -315,8 +315,9 @@ __device__ __forceinline__ void rest_terms(const DevConfig &cf, const uint32_t *
 // One warp per environment (boards of at most 512 cells, at most 16 rules),
 // on the one-warp rollout's layout and loop: each lane keeps every rule's
 // first four present terms in registers, and a step in which no rule
-// survives them has no raw match, so it is the standard quiet step.  A step
-// with survivors finishes their remaining terms into the registers (no
+// survives them has no raw match, so it is the standard quiet step; nor has a
+// rule whose tile terms pass nowhere on the board (tested once per board).  A
+// step with survivors finishes their remaining terms into the registers (no
 // writes yet: the raw matches), derives the suppressed set, keeps each
 // limited rule's largest keys, writes, and updates the board; no barrier.
 template <typename CellT, int NA, int RPW, bool SM>
@@ -451,6 +452,9 @@ __global__ void __launch_bounds__(128)
     const bool any_traj = rew_traj != nullptr || done_traj != nullptr || obs_traj != nullptr;
 
     int sum = 0;
+    // Rules tested on the current board and those that cannot match on it
+    // (env_dead_rules); warp-uniform, cleared when the board changes.
+    uint32_t known = 0, dead = 0;
     for (int s = 0; s < n_steps; ++s) {
         if (s > 0 && (s & (kActChunk / 2 - 1)) == 0)
             env_refill(actions, seed, env, s, n_steps, S.acts, S.ctl + 3);
@@ -467,7 +471,12 @@ __global__ void __launch_bounds__(128)
             }
             bits |= (a != 0u ? 1u : 0u) << k;
         }
-        const uint32_t live = __reduce_or_sync(0xffffffffu, bits);  // rules past their register terms
+        uint32_t live = __reduce_or_sync(0xffffffffu, bits);  // rules past their register terms
+        if (live & ~known) {  // rules live for the first time on this board
+            dead |= env_dead_rules<NA, SM>(cf, tab, S.vm, pbase, live & ~known);
+            known |= live;
+        }
+        live &= ~dead;  // no raw match possible: neither written nor inhibiting
         int rew = 0, changed = 0;
         if (live) {
             // raw matches: the rest of every live rule, into m (no writes)
@@ -508,6 +517,8 @@ __global__ void __launch_bounds__(128)
             t = r.x;
             goal_left = r.y;
             done = r.z;
+            known = 0;  // a new board
+            dead = 0;
         }
         sum += rew;
         // every read of this step's force is behind the step's last vote

@@ -1423,8 +1423,12 @@ rollout_fast_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
 // in their place), so a step in which no rule survives them is RPW x 4 shared
 // loads, one vote and the force copy: no barrier, no shared counter.  Rules
 // that do survive continue, one at a time, in a single inlined loop over the
-// remaining terms (four per vote, the next four fetched ahead).  A step with a
-// match combines the SET / CLEAR planes, tests the goal, resets when due and
+// remaining terms (four per vote, the next four fetched ahead).  A rule that
+// survives its register terms is first tested once per board on its tile
+// terms alone (env_dead_rules): one that passes nowhere on them is left out,
+// of the quiet loop's vote too, until the board changes, so that a rule stuck
+// a term short of a match does not cost a general step every step.  A step
+// with a match combines the SET / CLEAR planes, tests the goal, resets when due and
 // rebuilds the five force planes, all within the warp.
 
 // Per-lane register data of one rule: its valid anchors in this lane's words
@@ -1594,6 +1598,59 @@ static __device__ __noinline__ void env_refill(const uint8_t *actions, uint64_t 
     __syncwarp();
 }
 
+// Anchors of this lane's words at which every tile-channel term of rule k
+// passes on the current board (its force terms left out).  Only the force
+// terms change from one step to the next while the board stays as it is.
+template <int NA, bool SM>
+__device__ __forceinline__ void env_tile_terms(const DevConfig &cf, const uint32_t *tab, const uint32_t *vm_s,
+                                               uint32_t pbase, int k, uint32_t (&m)[NA])
+{
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+    const uint32_t plane_bytes = (uint32_t)cf.NWP * 8, force_lo = (uint32_t)cf.C * plane_bytes;
+    const uint4 h0 = ld4<SM>(tab + 4 + 8 * k);
+    const uint4 h1 = ld4<SM>(tab + 8 + 8 * k);
+    const uint32_t *vmr = vm_s + ((h1.z >> (8 * g)) & 0xffu) * cf.NW;
+#pragma unroll
+    for (int u = 0; u < NA; ++u) {
+        const int a = q + 8 * u;
+        m[u] = a < cf.NW ? vmr[a] : 0u;
+    }
+    for (uint32_t j = 0; j < h0.x + h0.y; ++j) {
+        const uint2 d = ld2<SM>(terms + (size_t)(h1.x + j) * 4 + g);
+        if (d.x - force_lo < plane_bytes)
+            continue;  // a force term
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            const uint2 w = lds2(pbase + d.x + 64 * u);
+            m[u] &= __funnelshift_r(w.x, w.y, d.y) ^ (uint32_t)((int32_t)d.y >> 31);
+        }
+    }
+}
+
+// Of `rules` (a warp-uniform bit set), the rules whose tile-channel terms pass
+// at no valid anchor of the current board (one warp): they cannot match again
+// before the board changes.  Not inlined, like env_step_outputs: it runs
+// once per rule and board.
+template <int NA, bool SM>
+static __device__ __noinline__ uint32_t env_dead_rules(DevConfig cf, const uint32_t *tab, const uint32_t *vm_s,
+                                                       uint32_t pbase, uint32_t rules)
+{
+    uint32_t dead = 0;
+    while (rules) {
+        const int k = __ffs(rules) - 1;
+        rules &= rules - 1;
+        uint32_t m[NA], any = 0;
+        env_tile_terms<NA, SM>(cf, tab, vm_s, pbase, k, m);
+#pragma unroll
+        for (int u = 0; u < NA; ++u)
+            any |= m[u];
+        if (!__any_sync(0xffffffffu, any != 0u))
+            dead |= 1u << k;
+    }
+    return dead;
+}
+
 template <typename CellT, int NA, int RPW, bool SM>
 __global__ void __launch_bounds__(128)
 rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
@@ -1728,6 +1785,17 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
 
     int sum = 0;
     uint32_t m[RPW][NA];  // anchors of each rule live after its register terms
+    // Rules already tested on the current board, and those of them that cannot
+    // match on it (env_dead_rules; warp-uniform, cleared when the board
+    // changes), and per rule a mask that is zero for such a rule, which the
+    // quiet loop applies to its vote.  Kernels with more than eight rules per
+    // lane run without the test: their registers are full already.
+    constexpr bool kDeadTest = RPW <= 8;
+    uint32_t known = 0, dead = 0;
+    uint32_t alive[kDeadTest ? RPW : 1];
+#pragma unroll
+    for (int k = 0; k < (kDeadTest ? RPW : 1); ++k)
+        alive[k] = 0xffffffffu;
     // Steps in which no rule survives its register terms and no reset is due:
     // t advances, the next step's force goes into the slot, nothing else
     // changes.  The loop is kept free of branches around rarely used code,
@@ -1745,7 +1813,7 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
 #pragma unroll
                 for (int u = 0; u < NA; ++u) {
                     m[k][u] = env_reg_terms(fr[k], u);
-                    anyall |= m[k][u];
+                    anyall |= m[k][u] & alive[kDeadTest ? k : 0];
                 }
             const bool reset_due = cf.auto_reset && !(goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps));
             if (__any_sync(0xffffffffu, anyall != 0u) || reset_due)
@@ -1803,14 +1871,24 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
                 }
                 bits |= (a != 0u ? 1u : 0u) << k;
             }
-            uint32_t live = __reduce_or_sync(0xffffffffu, bits);  // rules live past their register terms
+            const uint32_t raw = __reduce_or_sync(0xffffffffu, bits);  // rules live past their register terms
             const bool reset_due = cf.auto_reset && !(goal_left && (cf.max_steps <= 0 || t + 1 < cf.max_steps));
-            if (!live && !reset_due)
+            if (!raw && !reset_due)
                 break;  // a quiet step: back to the quiet loop
+            if (kDeadTest && (raw & ~known)) {  // rules live for the first time on this board
+                dead |= env_dead_rules<NA, SM>(cf, tab, S.vm, pbase, raw & ~known);
+                known |= raw;
+#pragma unroll
+                for (int k = 0; k < (kDeadTest ? RPW : 1); ++k)
+                    alive[k] = ((dead >> k) & 1u) ? 0u : 0xffffffffu;
+            }
+            uint32_t live = raw & ~dead;
+            if (!live && !reset_due)
+                break;  // only rules that cannot match: the quiet loop takes this step
 
             // ---- general step s: the rest of every live rule, writes
             int rew = 0, changed = 0;
-            {
+            if (live) {
                 int2 acc = make_int2(0, 0);
                 while (live) {
                     const int k = __ffs(live) - 1;
@@ -1844,6 +1922,11 @@ rollout_env_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const 
                 done = r.z;
                 f_next = lane < NW ? fplanes[a_next * NWP + lane] : make_uint2(0u, 0u);
                 sum += rew;
+                known = 0;  // a new board
+                dead = 0;
+#pragma unroll
+                for (int k = 0; k < (kDeadTest ? RPW : 1); ++k)
+                    alive[k] = 0xffffffffu;
             }
             // every read of this step's force is behind the step's last vote
             if (lane < NW)
