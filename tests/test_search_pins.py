@@ -3,8 +3,8 @@ its own forward model for best-first search; equal states keep the shallower
 node, and of equal states the higher reward): children equal to the pinned
 standard step, hashes equal to the pinned FNV-1a of the children's bytes, and
 closed forms of the search itself -- on an open floor the frontier after d
-rounds is exactly the ring of cells at Manhattan distance d (breadth-first
-layers), in a corridor of food the best reward after d rounds is the food
+iterations is exactly the ring of cells at Manhattan distance d (breadth-first
+layers), in a corridor of food the best reward after d iterations is the food
 within d cells -- plus the frontier's order and distinctness."""
 from __future__ import annotations
 
@@ -51,8 +51,8 @@ def test_expand_children_are_steps_and_hashes_are_fnv(key):
 
 def test_open_floor_search_is_breadth_first():
     """Only the move rule, an open floor, a beam wider than any layer: the
-    states are the player's cells, and round d keeps exactly the cells at
-    Manhattan distance d from the start that no earlier round reached."""
+    states are the player's cells, and iteration d keeps exactly the cells at
+    Manhattan distance d from the start that no earlier iteration reached."""
     H = W = 13
     g = _walled(H, W)
     y0, x0 = 6, 4
@@ -77,10 +77,10 @@ def test_open_floor_search_is_breadth_first():
 
 def test_food_corridor_best_reward():
     """A corridor with food at known distances right of the player: after d
-    rounds the best cumulative reward in the beam is the food within d cells
+    iterations the best cumulative reward in the beam is the food within d cells
     (moving onto food eats it, reward 1; Sec. 2.2.1).  Eating the last food
-    ends the episode (no goal left): that node stays in the beam of its round
-    but is not expanded, so one round later no node holds all the food."""
+    ends the episode (no goal left): that node stays in the beam of its iteration
+    but is not expanded, so one iteration later no node holds all the food."""
     W = 14
     g = _walled(3, W)
     g[1, 1] |= P
@@ -89,7 +89,7 @@ def test_food_corridor_best_reward():
         g[1, x] = G
     rules = wk.base_game_rules(4)[None]
     cfg = oracle.make_cfg(**_fields(1, 3, W))
-    last = food[-1] - 1  # rounds to reach the last food
+    last = food[-1] - 1  # iterations to reach the last food
     res = oracle.search(cfg, rules, g[None], last, 64)
     want = [sum(1 for x in food if x - 1 <= d) for d in range(1, last + 1)]
     np.testing.assert_array_equal(res["trace_best"][0], want)
