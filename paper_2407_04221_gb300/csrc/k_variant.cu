@@ -453,30 +453,50 @@ __global__ void __launch_bounds__(128)
 
     int sum = 0;
     // Rules tested on the current board and those that cannot match on it
-    // (env_dead_rules); warp-uniform, cleared when the board changes.
+    // (env_dead_rules; warp-uniform, cleared when the board changes), and per
+    // rule a mask that is zero for such a rule, applied to the step's first vote
+    // (kernels with more than eight rules per lane skip that vote: their
+    // registers are full already).
+    constexpr bool kQuietVote = RPW <= 8;
     uint32_t known = 0, dead = 0;
+    uint32_t alive[kQuietVote ? RPW : 1];
+#pragma unroll
+    for (int k = 0; k < (kQuietVote ? RPW : 1); ++k)
+        alive[k] = 0xffffffffu;
     for (int s = 0; s < n_steps; ++s) {
         if (s > 0 && (s & (kActChunk / 2 - 1)) == 0)
             env_refill(actions, seed, env, s, n_steps, S.acts, S.ctl + 3);
         const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
         uint32_t m[RPW][NA];
-        uint32_t bits = 0;
+        uint32_t anyall = 0;
 #pragma unroll
-        for (int k = 0; k < RPW; ++k) {
-            uint32_t a = 0;
+        for (int k = 0; k < RPW; ++k)
 #pragma unroll
             for (int u = 0; u < NA; ++u) {
                 m[k][u] = env_reg_terms(fr[k], u);
-                a |= m[k][u];
+                anyall |= m[k][u] & alive[kQuietVote ? k : 0];
             }
-            bits |= (a != 0u ? 1u : 0u) << k;
+        uint32_t live = 0;
+        if (!kQuietVote || __any_sync(0xffffffffu, anyall != 0u)) {  // else a quiet step
+            uint32_t bits = 0;
+#pragma unroll
+            for (int k = 0; k < RPW; ++k) {
+                uint32_t a = 0;
+#pragma unroll
+                for (int u = 0; u < NA; ++u)
+                    a |= m[k][u];
+                bits |= (a != 0u ? 1u : 0u) << k;
+            }
+            live = __reduce_or_sync(0xffffffffu, bits);  // rules past their register terms
+            if (live & ~known) {  // rules live for the first time on this board
+                dead |= env_dead_rules<NA, SM>(cf, tab, S.vm, pbase, live & ~known);
+                known |= live;
+#pragma unroll
+                for (int k = 0; k < (kQuietVote ? RPW : 1); ++k)
+                    alive[k] = ((dead >> k) & 1u) ? 0u : 0xffffffffu;
+            }
+            live &= ~dead;  // no raw match possible: neither written nor inhibiting
         }
-        uint32_t live = __reduce_or_sync(0xffffffffu, bits);  // rules past their register terms
-        if (live & ~known) {  // rules live for the first time on this board
-            dead |= env_dead_rules<NA, SM>(cf, tab, S.vm, pbase, live & ~known);
-            known |= live;
-        }
-        live &= ~dead;  // no raw match possible: neither written nor inhibiting
         int rew = 0, changed = 0;
         if (live) {
             // raw matches: the rest of every live rule, into m (no writes)
@@ -519,6 +539,9 @@ __global__ void __launch_bounds__(128)
             done = r.z;
             known = 0;  // a new board
             dead = 0;
+#pragma unroll
+            for (int k = 0; k < (kQuietVote ? RPW : 1); ++k)
+                alive[k] = 0xffffffffu;
         }
         sum += rew;
         // every read of this step's force is behind the step's last vote
