@@ -84,3 +84,32 @@ def test_valid_anchor_rules_by_hand():
     # 1x1: 4 rotations x 24 anchors; 2x3 on a 4x6 board: rotations 0, 2 have
     # (4-2+1) x (6-3+1) anchors, rotations 1, 3 (3x2) have (4-3+1) x (6-2+1)
     assert bench.valid_anchor_rules(wl, rules) == 4 * 24 + 2 * 12 + 2 * 10
+
+
+def test_profile_traffic_follows_the_kernel_source(tmp_path, monkeypatch):
+    """The bench line reports a profile's DRAM traffic only while the kernel
+    source hashes to the value recorded with the capture."""
+    import hashlib
+    from types import SimpleNamespace
+
+    src = tmp_path / "kernel.cu"
+    src.write_text("__global__ void k() {}\n")
+    digest = hashlib.sha256(src.read_bytes()).hexdigest()
+    monkeypatch.setattr(bench, "PROFILE_DIR", str(tmp_path))
+    wl = SimpleNamespace(name="toy")
+    prof = tmp_path / "k_toy.md"
+    prof.write_text(f"kernel_source_sha256: {digest[:16]}\ndram_bytes_per_launch: 12345\n")
+    assert bench.profile_traffic("k", wl, str(src)) == 12345.0
+    src.write_text("__global__ void k() { /* changed */ }\n")
+    assert bench.profile_traffic("k", wl, str(src)) is None
+    assert bench.profile_traffic("missing", wl, str(src)) is None
+
+
+def test_committed_profiles_name_their_kernel_sources():
+    """Every committed profile with a traffic figure records a source hash."""
+    import glob
+    import re
+    for path in glob.glob(os.path.join(bench.PROFILE_DIR, "*.md")):
+        text = open(path).read()
+        if "dram_bytes_per_launch:" in text:
+            assert re.search(r"kernel_source_sha256:\s*[0-9a-f]{16}", text), path
