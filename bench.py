@@ -1,16 +1,20 @@
 """Benchmark: batched Autoverse environment steps on one GB300 (per process).
 
-Default workload: 1024 envs, 16x16 boards, 8 tile channels, 8 rules of 3x3 in
-4 rotations each, per-env rule tables, 1000 fused steps per launch
-(av_rollout).  One benchmark step = one launch = 1024 x 1000 env-steps.
+Default workload (config 3, the RL training shape): 16,384 envs, 16x16 boards,
+10 tile channels, 12 rules per env of 1x2 / 1x3 / 3x3 in 4 rotations each,
+2000 fused steps per launch (av_rollout) writing the observation, reward and
+done flag of every step (16.9 GB per launch), done at no goal tile or t = 200
+with auto-reset.  One benchmark step = one launch = 16,384 x 2000 env-steps.
+The line also carries an `extra` entry for the 64x64 workload (config 5).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--config 2|3|5] [--seed S]
+                    [--config 1|2|3|4|5|6] [--single-step] [--seed S]
 
 Prints one JSON line.  Under torchrun (N > 1) every rank runs its own replica
 of the workload (envs never interact: no data-path collective); the timing is
 the max over ranks and `value` counts the env-steps of all ranks.
 
+--single-step times av_step (one launch per step) on the workload's shape.
 --impl reference times the CPU oracle (the slow, literal restatement of the
 paper's rule semantics) on this machine's host cores, on a bounded sample of
 the same workload; only rank 0 runs it.
@@ -39,8 +43,9 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "kernels.cuh")
 PROFILE_DIR = os.path.join(ROOT, "profiles")
 # rollout kernel launched for each av_rollout_path value
 KERNEL_NAMES = {1: "rollout_kernel", 2: "rollout_fast_kernel", 3: "rollout_env_warp_kernel",
-                4: "rollout_variant_kernel", 5: "rollout_band_kernel"}
+                4: "rollout_variant_kernel", 5: "rollout_band_kernel", 6: "rollout_memo_kernel"}
 VARIANT_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_variant.cu")
+MEMO_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_memo_impl.cuh")
 BAND_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_band.cu")
 
 
@@ -288,7 +293,7 @@ def run_reference(args, wl):
     line = {
         "impl": "reference", "metric": "env-steps/s", "value": value, "unit": "env-steps/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
         "data": "synthetic",
         "config": dict(config_dict(wl, sample=n), **({"workload": VariantName(wl).name,
                                                        "variant": bench_variant(wl)} if args.variant else {})),
@@ -306,30 +311,122 @@ def config_dict(wl, sample=None):
     full = wk.WORKLOADS[wl.key]
     name = wl.name if (wl.batch, wl.steps) == (full.batch, full.steps) else \
         f"{wl.name}, smaller case: {wl.batch} envs x {wl.steps} steps"
+    if wl.base_game:
+        name += " (rules 0-1 of each table: the maze game's 1x2 move and eat rules, not random 3x3)"
+    l2 = "flushed (256 MiB write) between timed launches"
+    if wl.trajectory:
+        gb = wl.batch * wl.steps * traj_bytes_per_env_step(wl) / 1e9
+        l2 = f"trajectory outputs ({gb:.1f} GB per launch) far exceed L2; also flushed (256 MiB write)" \
+             " between timed launches"
     d = {"workload": name, "batch": wl.batch, "H": wl.H,
          "W": wl.W, "tile_channels": wl.C, "rules": wl.n_rules, "rotations": 4,
          "pattern_sizes": [f"{h}x{w}" for h, w in wl.shapes],
          "fused_steps_per_launch": wl.steps, "per_env_rules": bool(wl.rules_per_env),
          "trajectory_outputs": wl.trajectory,
-         "l2": "flushed (256 MiB write) between timed launches", "parallelism": "replicas"}
+         "l2": l2, "parallelism": "replicas"}
+    if wl.max_steps or wl.auto_reset:
+        d["done"] = f"no goal tile left or t = {wl.max_steps}" + (", auto-reset" if wl.auto_reset else "")
     if sample:
         d["sample_envs"] = sample
     return d
 
 
 # ------------------------------------------------------------------ ours
-def run_ours(args, wl):
+def popcount(a: np.ndarray) -> np.ndarray:
+    a = a.astype(np.uint64)
+    c = np.zeros(a.shape, np.int64)
+    for b in range(32):
+        c += ((a >> np.uint64(b)) & np.uint64(1)).astype(np.int64)
+    return c
+
+
+def row_basis_ops(wl: wk.Workload, rules: np.ndarray) -> float:
+    """Full-evaluation op count of one env-step on the basis the hot-path scope
+    table uses: every rule rotation tests each input term (a present or absent
+    (position, channel) entry) and ORs each output entry once per valid anchor
+    ROW (one op per row of anchors), averaged over the environments' tables."""
+    h = rules["h"].astype(np.int64)
+    w = rules["w"].astype(np.int64)
+    entries = (popcount(rules["present"]).sum(-1) + popcount(rules["absent"]).sum(-1) +
+               popcount(rules["set"]).sum(-1) + popcount(rules["clear"]).sum(-1))
+    rows_a = np.clip(wl.H - h + 1, 0, None) * (wl.W - w + 1 > 0)  # rotations 0, 2
+    rows_b = np.clip(wl.H - w + 1, 0, None) * (wl.W - h + 1 > 0)  # rotations 1, 3
+    return float((entries * (2 * rows_a + 2 * rows_b)).sum(-1).mean())
+
+
+def traj_bytes_per_env_step(wl: wk.Workload) -> int:
+    """Algorithmic HBM bytes of one env-step of a trajectory rollout: the
+    observation (the board's canonical bytes), the int32 reward, the done byte."""
+    return wl.H * wl.W * wl.cell_bytes + 4 + 1
+
+
+def profile_field(kernel: str, wl, field: str, src: str = KERNEL_SRC) -> float | None:
+    """A machine-readable figure of the committed ncu summary of this kernel on
+    this workload, if the summary was taken on the current kernel source."""
+    try:
+        text = open(profile_path(kernel, wl)).read()
+    except OSError:
+        return None
+    m = re.search(r"kernel_source_sha256:\s*([0-9a-f]{16,64})", text)
+    t = re.search(field + r":\s*([0-9.eE+]+)", text)
+    if not m or not t:
+        return None
+    cur = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    return float(t.group(1)) if cur.startswith(m.group(1)) else None
+
+
+def kernel_source(path: int, av) -> str:
+    """The source file of the rollout kernel for an av_rollout_path value."""
+    if path == av.AV_PATH_MEMO:
+        return MEMO_SRC
+    if path == av.AV_PATH_VARIANT:
+        return VARIANT_SRC
+    if path == av.AV_PATH_BAND:
+        return BAND_SRC
+    return KERNEL_SRC
+
+
+def measure_activity(av, fields, rules, cum, wl, seed, dev, budget_bytes: int = 2 << 30) -> dict:
+    """How much the rules do on this workload, counted on the GPU by the library
+    itself (outside any timed region): one launch from the reset boards with the
+    timed launches' first action seed, on a copy of the rule tables whose
+    rewards are all 1, so that a step's reward is its number of rule
+    applications ((rule, rotation, anchor) matches).  Envs beyond what a
+    `budget_bytes` trajectory holds are left out (the first envs are kept)."""
+    import torch
+    per_env = wl.steps * wl.H * wl.W * wl.cell_bytes
+    n = max(1, min(wl.batch, budget_bytes // max(per_env, 1)))
+    r1 = rules.copy()
+    r1["reward"] = 1
+    if wl.rules_per_env:
+        r1 = r1[:n]
+    f = dict(fields, batch=n)
+    c1 = cum[:n] if (cum is not None and cum.ndim == 2 and cum.shape[0] == wl.batch) else cum
+    e = av.Env(f, r1, c1, device=dev)
+    s = wk.seeds(seed)
+    g0 = e.reset(s["reset"]).clone()
+    res = e.rollout(wl.steps, s["actions"], trajectory=True)
+    obs = res["obs"]
+    prev = torch.cat([g0[None], obs[:-1]], 0)
+    changed = (obs != prev).flatten(2).any(-1)
+    matches = res["rew"].double()
+    out = {"applications_per_env_step": float(matches.mean()),
+           "match_step_frac": float((res["rew"] > 0).double().mean()),
+           "board_change_frac": float(changed.double().mean()),
+           "done_frac": float(res["done"].double().mean()),
+           "source": f"library, first launch from the reset boards, {n} of {wl.batch} envs x"
+                     f" {wl.steps} steps, rewards set to 1 on a copy of the tables"}
+    e.close()
+    return out
+
+
+def time_rollout(args, wl, rank, world, dev, steps, warmup, e2e: bool):
+    """Times `steps` av_rollout launches of workload wl (after `warmup`), L2
+    flushed between launches outside the events.  Returns the measurements and
+    the handle's setup (rules, cum, fields, seed, env)."""
     import torch
 
     import paper_2407_04221_gb300 as av
-
-    rank, world, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
-    dev = torch.device("cuda", local if world > 1 else 0)
-    torch.cuda.set_device(dev)
     seed = args.seed + 1000 * rank
     _, rules, cum = wk.make(wl, seed)
     fields = wk.config_fields(wl)
@@ -352,8 +449,218 @@ def run_ours(args, wl):
         obs, rew, done = traj if traj else (None, None, None)
         av.av_rollout(env.h, wl.steps, s["actions"] + 7919 * i, obs, rew, done, rew_sum, stream)
 
-    for i in range(args.warmup):
+    for i in range(warmup):
         launch(i)
+    torch.cuda.synchronize(dev)
+    env.sync()
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    sampler = ClockSampler(torch.cuda.current_device() if world == 1 else local_index(dev))
+    sampler.start()
+    barrier()
+    sampler.mark_start()
+    t_wall = time.perf_counter()
+    for i in range(steps):
+        flush.fill_(i & 0xff)  # evict L2 between timed launches (outside the events)
+        starts[i].record(stream)
+        launch(warmup + i)
+        ends[i].record(stream)
+    barrier()
+    wall = time.perf_counter() - t_wall
+    sampler.mark_end()
+    clocks = sampler.stop()
+    env.sync()
+    ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
+    kernel_ms = sum(ms) / len(ms)
+    total_ms = max_over_ranks(sum(ms), world, dev)
+    out = dict(rules=rules, cum=cum, fields=fields, seed=seed, env=env, std_path=std_path,
+               kernel_ms=kernel_ms, total_ms=total_ms, wall=wall, clocks=clocks, g0=g0)
+    if e2e:
+        # the same launch through host buffers (pinned), copies timed
+        host_in = g0.cpu().pin_memory()
+        host_out = torch.empty(wl.batch, dtype=torch.int32).pin_memory()
+        dev_in = torch.empty_like(g0)
+        e2e_steps = max(3, min(steps, 20))
+        barrier()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(e2e_steps):
+            dev_in.copy_(host_in, non_blocking=True)
+            av.av_set_state(env.h, dev_in, None, False, stream)
+            launch(10_000 + i)
+            host_out.copy_(rew_sum, non_blocking=True)
+        e1.record(stream)
+        barrier()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
+        out["e2e"] = {"value": wl.batch * wl.steps * world / (e2e_ms / 1e3), "unit": "env-steps/s",
+                      "h2d_bytes_per_step": int(host_in.numel() * host_in.element_size()),
+                      "d2h_bytes_per_step": int(host_out.numel() * host_out.element_size())}
+    del traj, flush
+    return out
+
+
+def local_index(dev) -> int:
+    return dev.index if dev.index is not None else 0
+
+
+def rollout_roofline(av, wl, m, sm_mhz) -> dict:
+    """Roofline of the rollout kernel that ran: HBM for trajectory workloads
+    (the observation stream), integer issue otherwise."""
+    peaks = measured_peaks()
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    path = av.av_rollout_path(m["env"].h)
+    kernel = KERNEL_NAMES[path]
+    if path == av.AV_PATH_VARIANT and wl.key in (1, 2):
+        kernel = "rollout_variant_warp_kernel"  # variants on the one-warp layout
+    pw = VariantName(wl) if path == av.AV_PATH_VARIANT else wl
+    src = kernel_source(path, av)
+    env_steps = wl.batch * wl.steps
+    kernel_s = m["kernel_ms"] / 1e3
+    ops = row_basis_ops(wl, m["rules"])
+    peak_ops = SM_COUNT_GB300 * INT_LANES_PER_SM * sm_max * 1e6 / 1e9  # Gop/s
+    inst = profile_field(kernel, pw, "warp_instructions_per_launch", src)
+    clock = (sm_mhz or sm_max) * 1e6
+    alu = {"achieved": ops * env_steps / kernel_s / 1e9, "peak": peak_ops, "unit": "Gop/s",
+           "frac": ops * env_steps / kernel_s / 1e9 / peak_ops, "ops_per_env_step": ops,
+           "ops_basis": "full evaluation, one op per (rule rotation, input or output entry,"
+                        " valid anchor row); the kernels evaluate far less (early exit, and"
+                        " the memoising rollout evaluates a (board, action) pair once), so this"
+                        " ratio is a full-evaluation equivalent, not a utilisation",
+           "peak_from": f"{SM_COUNT_GB300} SMs x {INT_LANES_PER_SM} int32 lanes/clk"
+                        f" x {sm_max:.0f} MHz (sm_max_mhz of measured peaks); the LOP3 issue"
+                        " probe measured 76 of the 128 lanes/clk",
+           "issue_util": (inst / (SM_COUNT_GB300 * 4 * clock * kernel_s)) if inst else None,
+           "issue_util_basis": "ncu warp instructions of one launch (committed profile, scaled to"
+                               " this launch by env-steps) / (152 SMs x 4 schedulers x median SM"
+                               " clock x launch time)"}
+    if wl.batch == 1:
+        alu["note"] = ("one environment: the launch is bound by the latency of one CTA, so the"
+                       " fraction says nothing about the kernel's use of the GPU")
+    if wl.trajectory:
+        bpes = traj_bytes_per_env_step(wl)
+        peak = float(peaks.get("hbm_gbs", 6723.0))
+        achieved = bpes * env_steps / kernel_s / 1e9
+        return {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": profile_traffic(kernel, pw, src),
+                "kernel": kernel, "bytes_per_env_step": bpes,
+                "bytes_basis": "observation (board bytes) + int32 reward + done byte per env-step"
+                               " (boards in and out once per launch not counted)",
+                "peak_from": "hbm_gbs of measured peaks (copy bandwidth)", "alu": alu}
+    out = {"bound": "alu", "achieved": alu["achieved"], "peak": peak_ops, "unit": "Gop/s",
+           "frac": alu["frac"], "traffic": profile_traffic(kernel, pw, src), "kernel": kernel,
+           "ops_per_env_step": ops, "ops_basis": alu["ops_basis"], "peak_from": alu["peak_from"],
+           "issue_util": alu["issue_util"], "issue_util_basis": alu["issue_util_basis"]}
+    if "note" in alu:
+        out["note"] = alu["note"]
+    return out
+
+
+def run_ours(args, wl):
+    import torch
+
+    import paper_2407_04221_gb300 as av
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    m = time_rollout(args, wl, rank, world, dev, args.steps, args.warmup, e2e=True)
+    value = wl.batch * wl.steps * args.steps * world / (m["total_ms"] / 1e3)
+    activity = None
+    if rank == 0 and not args.variant:
+        activity = measure_activity(av, m["fields"], m["rules"], m["cum"], wl, m["seed"], dev)
+    extra = {}
+    if world == 1 and args.extra and wl.key == 3 and args.batch == 0 and args.fused_steps == 0:
+        wl5 = workload_for(5)
+        m5 = time_rollout(args, wl5, rank, world, dev, min(args.steps, 10), 3, e2e=False)
+        v5 = wl5.batch * wl5.steps * min(args.steps, 10) / (m5["total_ms"] / 1e3)
+        sm5 = (m5["clocks"] or {}).get("sm_mhz")
+        extra[wl5.name] = {
+            "value": v5, "unit": "env-steps/s", "steps": min(args.steps, 10), "warmup": 3,
+            "ms_per_step": m5["total_ms"] / min(args.steps, 10),
+            "config": config_dict(wl5),
+            "cell_rule_updates_per_s": v5 * wl5.H * wl5.W * wl5.n_rules * 4,
+            "roofline": rollout_roofline(av, wl5, m5, sm5),
+            "activity": measure_activity(av, m5["fields"], m5["rules"], m5["cum"], wl5, m5["seed"], dev),
+            "clocks": m5["clocks"]}
+        m5["env"].close()
+
+    if rank == 0:
+        sm_mhz = (m["clocks"] or {}).get("sm_mhz")
+        line = {
+            "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": m["total_ms"] / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+            "data": "synthetic",
+            "config": dict(config_dict(wl), **({"workload": VariantName(wl).name,
+                                                "variant": bench_variant(wl)} if args.variant else {})),
+            "cell_rule_updates_per_s": value * wl.H * wl.W * wl.n_rules * 4,
+            "valid_anchor_rule_tests_per_s": value * valid_anchor_rules(wl, m["rules"]),
+            "e2e": m["e2e"],
+            "roofline": rollout_roofline(av, wl, m, sm_mhz),
+            "gpu_launches": args.steps,
+            "wall_s_timed_region": m["wall"],
+        }
+        if activity:
+            line["activity"] = activity
+        if m["clocks"]:
+            line["clocks"] = m["clocks"]
+        if world == 1 and not args.no_cpu_baseline:
+            import oracle
+            cfg = oracle.make_cfg(**m["fields"])
+            line["cpu_baseline"] = cpu_baseline(wl, m["rules"], m["cum"], cfg, m["seed"],
+                                                variant=bench_variant(wl) if args.variant else None)
+        if extra:
+            line["extra"] = extra
+        print(json.dumps(line))
+    m["env"].close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def run_single_step(args, wl):
+    """One benchmark step = one av_step over the workload's batch: one kernel
+    launch, the boards read and written once, obs / reward / done written to
+    caller buffers, actions read from a device buffer (seeded, uniform 0..4,
+    a new row each step).  L2 flushed between timed launches."""
+    import torch
+
+    import paper_2407_04221_gb300 as av
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    seed = args.seed + 1000 * rank
+    _, rules, cum = wk.make(wl, seed)
+    fields = wk.config_fields(wl)
+    env = av.Env(fields, rules, cum, device=dev)
+    s = wk.seeds(seed)
+    env.reset(s["reset"])
+    n_act = args.warmup + args.steps
+    acts = torch.from_numpy(wk.actions(s["actions"], wl.batch, n_act)).to(dev)  # [n_act][B] uint8
+    obs = env.boards(wl.batch)
+    rew = torch.zeros(wl.batch, dtype=torch.int32, device=dev)
+    done = torch.zeros(wl.batch, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    for i in range(args.warmup):
+        av.av_step(env.h, acts[i], obs, rew, done, stream)
     torch.cuda.synchronize(dev)
     env.sync()
 
@@ -371,9 +678,9 @@ def run_ours(args, wl):
     sampler.mark_start()
     t_wall = time.perf_counter()
     for i in range(args.steps):
-        flush.fill_(i & 0xff)  # evict L2 between timed launches (outside the events)
+        flush.fill_(i & 0xff)
         starts[i].record(stream)
-        launch(args.warmup + i)
+        av.av_step(env.h, acts[args.warmup + i], obs, rew, done, stream)
         ends[i].record(stream)
     barrier()
     wall = time.perf_counter() - t_wall
@@ -382,83 +689,74 @@ def run_ours(args, wl):
     env.sync()
     ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
     kernel_ms = sum(ms) / len(ms)
-    total_ms = sum(ms)
-    total_ms = max_over_ranks(total_ms, world, dev)
-    env_steps = wl.batch * wl.steps * args.steps * world
-    value = env_steps / (total_ms / 1e3)
+    total_ms = max_over_ranks(sum(ms), world, dev)
+    value = wl.batch * args.steps * world / (total_ms / 1e3)
 
-    # ---- e2e: the same launch through host buffers (pinned), copies timed
-    host_in = g0.cpu().pin_memory()
-    host_out = torch.empty(wl.batch, dtype=torch.int32).pin_memory()
-    dev_in = torch.empty_like(g0)
-    e2e_steps = max(3, min(args.steps, 20))
+    # e2e: actions in from pinned host memory, rewards and done flags back
+    host_a = acts[: min(20, n_act)].cpu().pin_memory()
+    host_r = torch.empty(wl.batch, dtype=torch.int32).pin_memory()
+    host_d = torch.empty(wl.batch, dtype=torch.uint8).pin_memory()
+    dev_a = torch.empty_like(acts[0])
+    e2e_steps = max(3, min(args.steps, host_a.shape[0]))
     barrier()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(e2e_steps):
-        dev_in.copy_(host_in, non_blocking=True)
-        av.av_set_state(env.h, dev_in, None, False, stream)
-        launch(10_000 + i)
-        host_out.copy_(rew_sum, non_blocking=True)
+        dev_a.copy_(host_a[i], non_blocking=True)
+        av.av_step(env.h, dev_a, obs, rew, done, stream)
+        host_r.copy_(rew, non_blocking=True)
+        host_d.copy_(done, non_blocking=True)
     e1.record(stream)
     barrier()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    e2e_ms = max_over_ranks(e2e_ms, world, dev)
-    e2e_value = wl.batch * wl.steps * world / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world, dev)
 
     if rank == 0:
         peaks = measured_peaks()
-        sm_max = float(peaks.get("sm_max_mhz", 2070.0))
-        peak_ops = SM_COUNT_GB300 * INT_LANES_PER_SM * sm_max * 1e6 / 1e9  # Gop/s
-        ops = algorithmic_ops(wl, rules)
-        achieved = ops * wl.batch * wl.steps / (kernel_ms / 1e3) / 1e9
         path = av.av_rollout_path(env.h)
         kernel = KERNEL_NAMES[path]
-        if path == av.AV_PATH_VARIANT and std_path == av.AV_PATH_WARP:
-            kernel = "rollout_variant_warp_kernel"  # variants on the one-warp layout
-        traffic = (profile_traffic(kernel, VariantName(wl), VARIANT_SRC) if path == av.AV_PATH_VARIANT
-                   else profile_traffic(kernel, wl, BAND_SRC) if path == av.AV_PATH_BAND
-                   else profile_traffic(kernel, wl))
+        src = kernel_source(path, av)
+        sw = SingleStepName(wl)
+        board = wl.H * wl.W * wl.cell_bytes
+        bpes = 2 * board + 1 + 4 + 1
+        peak = float(peaks.get("hbm_gbs", 6723.0))
+        achieved = bpes * wl.batch / (kernel_ms / 1e3) / 1e9
+        traffic = profile_traffic(kernel, sw, src)
         line = {
             "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
             "data": "synthetic",
-            "config": dict(config_dict(wl), **({"workload": VariantName(wl).name,
-                                                "variant": bench_variant(wl)} if args.variant else {})),
-            "cell_rule_updates_per_s": value * wl.H * wl.W * wl.n_rules * 4,
-            "valid_anchor_rule_tests_per_s": value * valid_anchor_rules(wl, rules),
-            "e2e": {"value": e2e_value, "unit": "env-steps/s",
-                    "h2d_bytes_per_step": int(host_in.numel() * host_in.element_size()),
-                    "d2h_bytes_per_step": int(host_out.numel() * host_out.element_size())},
-            "roofline": {"bound": "alu", "achieved": achieved, "peak": peak_ops,
-                         "unit": "Gop/s", "frac": achieved / peak_ops,
-                         "traffic": traffic,
-                         "kernel": kernel,
-                         "ops_per_env_step": ops,
-                         "ops_basis": "full evaluation: every term and output entry of every"
-                                      " rule rotation at every valid anchor, one 32-bit word"
-                                      " op per 32 anchors; the kernels stop evaluating a rule"
-                                      " once no anchor is live, so frac can exceed 1",
-                         "peak_from": f"{SM_COUNT_GB300} SMs x {INT_LANES_PER_SM} int32 lanes/clk"
-                                      f" x {sm_max:.0f} MHz (sm_max_mhz of measured peaks)"},
+            "config": dict(config_dict(wl), workload=sw.name, fused_steps_per_launch=1,
+                           actions="seeded uniform 0..4 from a device buffer, one row per step",
+                           l2="flushed (256 MiB write) between timed launches"),
+            "e2e": {"value": wl.batch * world / (e2e_ms / 1e3), "unit": "env-steps/s",
+                    "h2d_bytes_per_step": wl.batch, "d2h_bytes_per_step": 5 * wl.batch},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": traffic, "kernel": kernel,
+                         "bytes_per_env_step": bpes,
+                         "bytes_basis": "board in + observation out + action + int32 reward + done"
+                                        " byte; the handle's own copy of the board written back and"
+                                        " the env's rule table (per-env tables, read every launch)"
+                                        " are extra traffic, counted in `traffic`",
+                         "traffic_per_env_step": traffic / wl.batch if traffic else None,
+                         "peak_from": "hbm_gbs of measured peaks (copy bandwidth)"},
             "gpu_launches": args.steps,
             "wall_s_timed_region": wall,
         }
         if clocks:
             line["clocks"] = clocks
-        if world == 1 and not args.no_cpu_baseline:
-            import oracle
-            cfg = oracle.make_cfg(**fields)
-            line["cpu_baseline"] = cpu_baseline(wl, rules, cum, cfg, seed,
-                                                variant=bench_variant(wl) if args.variant else None)
         print(json.dumps(line))
     env.close()
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
     return 0
+
+
+class SingleStepName:
+    """Profile naming for single-step launches of a workload."""
+    def __init__(self, wl):
+        self.name = f"{wl.name.replace('-traj', '')}-step"
 
 
 # ------------------------------------------------------------ search (config 4)
@@ -1150,7 +1448,12 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--config", type=int, default=2, choices=(2, 3, 4, 5, 6))
+    ap.add_argument("--config", type=int, default=3, choices=(1, 2, 3, 4, 5, 6))
+    ap.add_argument("--no-extra", dest="extra", action="store_false",
+                    help="config 3 only: skip the extra line for the 64x64 workload (config 5)")
+    ap.add_argument("--single-step", action="store_true",
+                    help="time av_step (one launch per step, obs / reward / done written) on the"
+                         " workload's shape instead of fused rollouts")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
@@ -1191,6 +1494,8 @@ def main(argv=None):
         return run_search_reference(args, wl) if args.impl == "reference" else run_search(args, wl)
     if args.impl == "reference":
         return run_reference(args, wl)
+    if args.single_step:
+        return run_single_step(args, wl)
     return run_ours(args, wl)
 
 

@@ -333,19 +333,22 @@ int av_sync(av_handle *h);
 int av_warnings(av_handle *h, uint32_t *bits);
 
 /* Which rollout kernel av_step / av_rollout launch for this handle:
- * AV_PATH_BLOCK (one CTA per environment), AV_PATH_FAST (several warps per
- * environment, boards of at most 512 cells and at most 64 rules) or
+ * AV_PATH_MEMO (boards of at most 512 cells, any rule count: one CTA per
+ * environment that evaluates each (board, action) pair once and repeats its
+ * outcome while the board stays unchanged), AV_PATH_BLOCK (one CTA per
+ * environment, every step evaluated; larger boards), AV_PATH_VARIANT when
+ * variant semantics are set (av_set_variant), or AV_PATH_BAND for boards of
+ * more than AV_MAX_SMEM_CELLS cells (one CTA per environment streams the
+ * board through shared memory in bands of rows).  AV_PATH_FAST (several warps
+ * per environment, boards of at most 512 cells and at most 64 rules) and
  * AV_PATH_WARP (one warp per environment, boards of at most 512 cells and at
- * most 16 rules), AV_PATH_VARIANT when variant semantics are set
- * (av_set_variant), or AV_PATH_BAND for boards of more than AV_MAX_SMEM_CELLS
- * cells (one CTA per environment streams the board through shared memory in
- * bands of rows).  The library picks the last of the first three that fits, except that rule sets
- * expected to keep matching on most steps (estimated by av_create from the
- * rules' leading present terms and the init_cum densities) take the block
- * kernel.  The environment variable AV_KERNEL_PATH=block|fast|warp, read by
- * av_create, forces one for tests and measurements.  Writes the path to
- * *path; AV_EINVAL for a null argument.  No GPU work. */
-enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3, AV_PATH_VARIANT = 4, AV_PATH_BAND = 5 };
+ * most 16 rules) step every environment every step; they run when the
+ * environment variable AV_KERNEL_PATH=block|fast|warp|memo, read by av_create,
+ * forces a path for tests and measurements.  Every path gives the same
+ * results.  Writes the path to *path; AV_EINVAL for a null argument.  No GPU
+ * work. */
+enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3, AV_PATH_VARIANT = 4, AV_PATH_BAND = 5,
+       AV_PATH_MEMO = 6 };
 int av_rollout_path(av_handle *h, int32_t *path);
 
 /* Static description of a status code. */

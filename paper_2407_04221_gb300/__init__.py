@@ -30,6 +30,7 @@ AV_MAX_WINDOW = 127
 AV_MAX_LIMIT = 255
 AV_PATH_VARIANT = 4
 AV_PATH_BAND = 5
+AV_PATH_MEMO = 6
 AV_MAX_SMEM_CELLS = 4096
 AV_SELECT_STATIC_MAX_HASHES = 1 << 21
 

@@ -467,7 +467,18 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     // per env); by default the library chooses.  AV_FAST_WARPS=8 runs the fast
     // rollout with 8 warps per env.
     if (const char *path = getenv("AV_KERNEL_PATH"))
-        cf.path = strcmp(path, "block") == 0 ? 1 : strcmp(path, "fast") == 0 ? 2 : strcmp(path, "warp") == 0 ? 3 : 0;
+        cf.path = strcmp(path, "block") == 0  ? 1
+                  : strcmp(path, "fast") == 0 ? 2
+                  : strcmp(path, "warp") == 0 ? 3
+                  : strcmp(path, "memo") == 0 ? 4
+                                              : 0;
+    // AV_MEMO_STAGE=1 or 0: the memoising rollout copies the rule tables into
+    // shared memory, or reads them through the L1 cache (default: decided by size).
+    if (const char *ms = getenv("AV_MEMO_STAGE"))
+        cf.memo_stage = atoi(ms) ? 1 : 2;
+    // AV_MEMO_WARPS=1|2|4: warps per environment of the memoising rollout.
+    if (const char *mw = getenv("AV_MEMO_WARPS"))
+        cf.memo_warps = atoi(mw);
     if (const char *fw = getenv("AV_FAST_WARPS"))
         cf.fast_warps = atoi(fw) == 8 ? 8 : 4;
     h->grid_bytes = (size_t)cf.HW * cf.cell_bytes;
@@ -925,6 +936,7 @@ int av_rollout_path(av_handle *h, int32_t *path)
         return AV_EINVAL;
     *path = h->large                   ? AV_PATH_BAND
             : h->variant_on            ? AV_PATH_VARIANT
+            : use_memo_rollout(h->cf)  ? AV_PATH_MEMO
             : use_env_warp_rollout(h->cf) ? AV_PATH_WARP
             : use_fast_rollout(h->cf)     ? AV_PATH_FAST
                                           : AV_PATH_BLOCK;

@@ -1,0 +1,628 @@
+// k_memo_impl.cuh -- fused rollout that remembers, for the board in hand, the
+// outcome of each action it has taken on it; included by k_memo_u8.cu and
+// k_memo_u16.cu (boards of at most 16 plane words, any rule count).
+//
+// A step's result is a function of the board, the action and the step
+// counter (Sec. 2.1: the rules are matched on the current board; the action
+// enters only as the force tiles next to the player).  While a board stays
+// unchanged, the step with action a always pays the same reward, writes the
+// same SET / CLEAR bits and leaves the same goal count.  One CTA runs one
+// environment and keeps, per action, the outcome of that step on the current
+// board once it has been computed: its reward and whether a goal tile is left
+// (an action whose step changes the board changes it at once, so the actions
+// remembered are the ones that leave it as it is).  A launch walks its steps
+// 32 at a time, one step per lane: every lane looks up its step's action, and
+// the first step whose action has no outcome yet, or that triggers an
+// auto-reset, ends the run of steps that merely repeat the board.  Those steps
+// write their rewards, done flags and observations (the board's canonical
+// bytes, held in registers) at once, the CTA's warps taking turns.  The step
+// that ended the run is evaluated by all warps together (every rule on the
+// board with that action's force, as the step-by-step kernels do, the rules
+// shared out among the warps); if it leaves the board unchanged its outcome is
+// remembered and the walk goes on, else its flips are applied (or the initial
+// map restored) and everything remembered is dropped.  No outcome is guessed:
+// each is computed once per board and action, so results are exactly those of
+// the step-by-step kernels.  Every warp runs the same walk on the same data
+// (the action draws, the remembered outcomes and the step counter are the same
+// in each), so all of them reach each block barrier together.
+#pragma once
+
+#include "launch.h"
+
+namespace av {
+
+constexpr int kMemoLead = 4;  // leading terms of each rule tested for all rules at once
+
+// Shared memory of one environment (one CTA): the valid-anchor and column
+// masks; tile planes 0..C-1, the force of the action being evaluated (plane
+// C) and an all-zero plane C+1 (padding terms read it as absent and pass),
+// doubled; SET and CLEAR planes (SET becomes the flip planes of the evaluated
+// step); the initial map's planes (flat); per rule its two header words
+// (uint4 each) and its first kMemoLead terms in each rotation; the board's
+// canonical bytes; per-warp reductions; the whole rule table when staged.
+struct MemoLayout {
+    size_t vm, masks, planes, setp, clrp, basep, hdr, lead, cells, red, rules, total;
+};
+
+__host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool staged)
+{
+    MemoLayout L;
+    const size_t pw = (size_t)cf.C * cf.NW * 4;  // one plane set, bytes
+    L.vm = 0;
+    L.masks = align16((size_t)kShapes * cf.NW * 4);
+    L.planes = align16(L.masks + (size_t)3 * cf.NW * 4);
+    L.setp = align16(L.planes + (size_t)(cf.C + 2) * cf.NWP * 8);
+    L.clrp = align16(L.setp + pw);
+    L.basep = align16(L.clrp + pw);
+    L.hdr = align16(L.basep + pw);
+    L.lead = align16(L.hdr + (size_t)cf.R * 32);
+    L.cells = align16(L.lead + (size_t)cf.R * 4 * kMemoLead * 8);
+    L.red = align16(L.cells + (size_t)cf.HW * cf.cell_bytes);
+    L.rules = align16(L.red + 16 * 4);
+    L.total = align16(L.rules + (staged ? (size_t)cf.rule_words * 4 : 0));
+    return L;
+}
+
+// Warps per environment (CTA): AV_MEMO_WARPS=1|2|4, read by av_create, else 2.
+inline int memo_warps(const DevConfig &cf) { return cf.memo_warps == 1 || cf.memo_warps == 4 ? cf.memo_warps : 2; }
+
+// Whether the whole rule table is copied into shared memory: when the
+// environment's region with it still lets as many environments share an SM
+// as the register budget does (32 warps of 64 registers per thread), else the
+// table is read through the L1 cache, and only for rules that pass their
+// leading terms.  AV_MEMO_STAGE=1 (copy) or 0 (do not), read by av_create,
+// forces the choice for measurements.
+inline bool memo_staged(const DevConfig &cf)
+{
+    if (cf.rule_words <= 0 || cf.memo_stage == 2)
+        return false;
+    const size_t total = memo_layout(cf, true).total;
+    if (cf.memo_stage == 1)
+        return total <= (size_t)kDynSmemLimit;
+    return total * (size_t)(32 / memo_warps(cf)) <= (size_t)224 * 1024;
+}
+
+// This lane's share of a board's canonical bytes to dst (global): 16-byte
+// stores (mode 0: the board size and dst 16-byte aligned), 4-byte stores
+// (mode 1) or single bytes (mode 2); nothing at or past nbytes.
+template <int NV>
+__device__ __forceinline__ void memo_store(unsigned char *dst, const uint32_t (&v)[4 * NV], int nbytes, int mode)
+{
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+        const int off = 16 * (lane + 32 * j);
+        if (off >= nbytes)
+            continue;
+        if (mode == 0) {
+            *reinterpret_cast<uint4 *>(dst + off) = make_uint4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int o = off + 4 * i;
+                if (mode == 1) {
+                    if (o < nbytes)
+                        *reinterpret_cast<uint32_t *>(dst + o) = v[4 * j + i];
+                } else {
+                    for (int k = 0; k < 4 && o + k < nbytes; ++k)
+                        dst[o + k] = (unsigned char)(v[4 * j + i] >> (8 * k));
+                }
+            }
+        }
+    }
+}
+
+__host__ __device__ inline int memo_store_mode(const void *p, int nbytes)
+{
+    const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+    if (nbytes % 16 == 0 && a % 16 == 0)
+        return 0;
+    if (nbytes % 4 == 0 && a % 4 == 0)
+        return 1;
+    return 2;
+}
+
+// Shared memory of one environment, as pointers.
+struct MemoSmem {
+    uint2 *planes;
+    uint32_t *setp, *clrp, *basep, *vm, *masks, *cells;
+    int *red;           // [w] reward of warp w's rules; [8] a bit flips; [9] a goal tile is left
+    const uint4 *hdr;   // [R][2]: (n_present, n_absent, n_out, reward), (first term, first output, shapes, 0)
+    const uint2 *lead;  // [R][4 rotations][kMemoLead] term descriptors
+};
+
+// Anchors of this lane's words at which rule r's first kMemoLead terms pass
+// (the valid-anchor mask of the lane's rotation ANDed with each term's
+// shifted plane word, absent terms complemented).
+template <int NA>
+__device__ __forceinline__ void memo_lead(const DevConfig &cf, const MemoSmem &S, uint32_t pbase, int r,
+                                          uint32_t (&m)[NA])
+{
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    const uint32_t shapes = S.hdr[2 * r + 1].z;
+    const uint32_t *vmr = S.vm + ((shapes >> (8 * g)) & 0xffu) * cf.NW;
+    const uint4 d01 = *reinterpret_cast<const uint4 *>(S.lead + (r * 4 + g) * kMemoLead);
+    const uint4 d23 = *reinterpret_cast<const uint4 *>(S.lead + (r * 4 + g) * kMemoLead + 2);
+    const uint32_t dx[4] = {d01.x, d01.z, d23.x, d23.z}, dy[4] = {d01.y, d01.w, d23.y, d23.w};
+#pragma unroll
+    for (int u = 0; u < NA; ++u) {
+        const int a = q + 8 * u;
+        uint32_t x = a < cf.NW ? vmr[a] : 0u;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint2 w = lds2(pbase + dx[j] + 64 * u);
+            x &= __funnelshift_r(w.x, w.y, dy[j]) ^ (uint32_t)((int32_t)dy[j] >> 31);
+        }
+        m[u] = x;
+    }
+}
+
+// One step of the board in S.planes with action `a`, by all NWARP warps of the
+// CTA: every rule in its four rotations as in the step-by-step kernels (warp w
+// takes rules w, w + NWARP, ...): the force plane of `a`, the leading terms of
+// the warp's rules, the remaining terms of those that pass them (four per
+// vote), the outputs of live matches ORed into SET / CLEAR; then the flip
+// planes (SET bits on clear cells, CLEAR bits on set cells) in place of
+// S.setp.  `n_terms` is the table's term count (its word 1).  Returns
+// (reward, bit 0: the step changes the board, bit 1: a goal tile is left
+// after it, always without a goal channel), the same in every thread.  Not
+// inlined: it runs once per board and action.
+template <int NA, bool SM, int NWARP>
+static __device__ __noinline__ int2 memo_step_eval(DevConfig cf, const uint32_t *tab, uint32_t n_terms, MemoSmem S,
+                                                   int a)
+{
+    constexpr int T = 32 * NWARP;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 3, q = lane & 7;
+    const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
+    for (int i = tid; i < cnw; i += T) {
+        S.setp[i] = 0u;
+        S.clrp[i] = 0u;
+    }
+    if (tid < 16)
+        S.red[tid] = 0;
+    if (warp == NWARP - 1)
+        force_plane(cf, S.planes, S.masks, a);
+    __syncthreads();
+    const uint32_t pbase = (uint32_t)__cvta_generic_to_shared(S.planes) + q * 8;
+    // this warp's rules whose leading terms pass somewhere
+    uint32_t alive0 = 0, alive1 = 0;
+#pragma unroll 2
+    for (int r = warp; r < cf.R; r += NWARP) {
+        uint32_t m[NA], any = 0;
+        memo_lead<NA>(cf, S, pbase, r, m);
+#pragma unroll
+        for (int u = 0; u < NA; ++u)
+            any |= m[u];
+        if (any) {
+            if (r < 32)
+                alive0 |= 1u << r;
+            else
+                alive1 |= 1u << (r - 32);
+        }
+    }
+    alive0 = __reduce_or_sync(0xffffffffu, alive0);
+    alive1 = cf.R > 32 ? __reduce_or_sync(0xffffffffu, alive1) : 0u;
+    const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+    const uint4 *outs = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, n_terms));
+    const uint32_t pass_x = (uint32_t)(cf.C + 1) * NWP * 8;  // a term on the zero plane, read as absent
+    int rew = 0;
+    for (int k = 0; k < 2; ++k) {
+        uint32_t alive = k ? alive1 : alive0;
+        while (alive) {
+            const int r = 32 * k + __ffs(alive) - 1;
+            alive &= alive - 1;
+            uint32_t m[NA];
+            memo_lead<NA>(cf, S, pbase, r, m);
+            const uint4 h0 = S.hdr[2 * r], h1 = S.hdr[2 * r + 1];
+            const uint32_t nt = h0.x + h0.y;
+            const uint2 *tp = terms + (size_t)h1.x * 4 + g;
+            bool live = true;
+            for (uint32_t t = kMemoLead; live && t < nt; t += 4) {
+                uint2 d[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    d[j] = t + j < nt ? ld2<SM>(tp + 4 * (t + j)) : make_uint2(pass_x, kTermAbsent);
+                uint32_t any = 0;
+#pragma unroll
+                for (int u = 0; u < NA; ++u) {
+                    uint32_t x = m[u];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const uint2 w = lds2(pbase + d[j].x + 64 * u);
+                        x &= __funnelshift_r(w.x, w.y, d[j].y) ^ (uint32_t)((int32_t)d[j].y >> 31);
+                    }
+                    m[u] = x;
+                    any |= x;
+                }
+                live = __any_sync(0xffffffffu, any != 0u);
+            }
+            if (!live)
+                continue;
+            uint32_t cnt = 0;
+#pragma unroll
+            for (int u = 0; u < NA; ++u)
+                cnt += __popc(m[u]);
+            if (cnt) {  // this lane's live anchors pay and write
+                rew += (int)h0.w * (int)cnt;
+                const uint4 *op = outs + (size_t)h1.y * 4 + g;
+                for (uint32_t o = 0; o < h0.z; ++o) {
+                    const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
+#pragma unroll
+                    for (int u = 0; u < NA; ++u) {
+                        if (!m[u])
+                            continue;
+                        const int w0 = q + 8 * u + (int)ov.x;
+                        const uint32_t lo = m[u] << ov.y;
+                        const uint32_t hi = ov.y ? (m[u] >> (32u - ov.y)) : 0u;
+                        scatter_bits(S.setp, ov.z, NW, w0, lo, hi);
+                        scatter_bits(S.clrp, ov.w, NW, w0, lo, hi);
+                    }
+                }
+            }
+            __syncwarp();
+        }
+    }
+    rew = __reduce_add_sync(0xffffffffu, rew);
+    if (lane == 0)
+        S.red[warp] = rew;
+    __syncthreads();  // every warp's SET / CLEAR bits and reward
+    uint32_t any = 0, goal = 0;
+    for (int i = tid; i < cnw; i += T) {
+        const int c = i / NW, w = i - c * NW;
+        const uint32_t d = S.planes[c * NWP + w].x;
+        const uint32_t f = (d & S.clrp[i]) | (~d & S.setp[i]);  // a bit changes where a match asks for it
+        S.setp[i] = f;
+        any |= f;
+        if (c == cf.ch_goal)
+            goal |= d ^ f;
+    }
+    any = __any_sync(0xffffffffu, any != 0u);
+    goal = __any_sync(0xffffffffu, goal != 0u);
+    if (lane == 0 && any)
+        atomicOr(S.red + 8, 1);
+    if (lane == 0 && goal)
+        atomicOr(S.red + 9, 1);
+    __syncthreads();  // the flip planes and flags
+    int total = 0;
+#pragma unroll
+    for (int w = 0; w < NWARP; ++w)
+        total += S.red[w];
+    const int bits = (S.red[8] ? 1 : 0) | ((cf.ch_goal < 0 || S.red[9]) ? 2 : 0);
+    __syncthreads();  // every thread has read the reductions before they are reused
+    return make_int2(total, bits);
+}
+
+// The board after its step: planes ^= flip (all warps).
+template <int NWARP>
+static __device__ __noinline__ void memo_apply(DevConfig cf, uint2 *planes, const uint32_t *flip)
+{
+    const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
+    for (int i = threadIdx.x; i < cnw; i += 32 * NWARP) {
+        const uint32_t f = flip[i];
+        const int c = i / NW, w = i - c * NW;
+        if (f)
+            put_word(planes, NWP, c, w, planes[c * NWP + w].x ^ f);
+    }
+    __syncthreads();
+}
+
+// Auto-reset: the initial map's planes back into the tile planes (all warps).
+// Returns whether the board differed from the initial map (every thread).
+template <int NWARP>
+static __device__ __noinline__ int memo_restore(DevConfig cf, uint2 *planes, const uint32_t *basep)
+{
+    const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
+    int diff = 0;
+    for (int i = threadIdx.x; i < cnw; i += 32 * NWARP) {
+        const uint32_t b = basep[i];
+        const int c = i / NW, w = i - c * NW;
+        if (planes[c * NWP + w].x != b) {
+            diff = 1;
+            put_word(planes, NWP, c, w, b);
+        }
+    }
+    return __syncthreads_or(diff);
+}
+
+// The board's canonical bytes into `cells` (shared, a whole number of
+// 16-byte units, zero past the board) from the doubled tile planes (all
+// warps), then this lane's 16-byte units of them into v.
+template <typename CellT, int NV, int NWARP>
+__device__ __forceinline__ void memo_cells(const DevConfig &cf, const uint2 *planes, uint32_t *cells,
+                                           uint32_t (&v)[4 * NV])
+{
+    constexpr int kPer = 4 / (int)sizeof(CellT);  // cells per word
+    const int HW = cf.HW, NWP = cf.NWP;
+    const int n16 = (HW * (int)sizeof(CellT) + 15) / 16;
+    for (int k = threadIdx.x; k < 4 * n16; k += 32 * NWARP) {
+        const int p0 = k * kPer;
+        uint32_t x = 0;
+        if (p0 < HW) {
+            const int w = p0 >> 5, b = p0 & 31;  // a word's cells lie in one plane word
+            for (int c = 0; c < cf.C; ++c) {
+                const uint32_t y = planes[c * NWP + w].x >> b;
+                const uint32_t s = sizeof(CellT) == 1 ? ((y & 0xfu) * 0x00204081u) & 0x01010101u
+                                                      : ((y & 0x3u) * 0x00008001u) & 0x00010001u;
+                x |= s << c;
+            }
+        }
+        cells[k] = x;
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+        const int u = lane + 32 * j;
+        const uint4 x = u < n16 ? reinterpret_cast<const uint4 *>(cells)[u] : make_uint4(0u, 0u, 0u, 0u);
+        v[4 * j] = x.x;
+        v[4 * j + 1] = x.y;
+        v[4 * j + 2] = x.z;
+        v[4 * j + 3] = x.w;
+    }
+}
+
+// Fused rollout, one CTA of NWARP warps per environment; see the top of this
+// file.  With `actions` non-null the action of every step is actions[env]
+// (av_step, n_steps = 1); else step s draws draw(seed, 4, env, 0, s) mod 5.
+template <typename CellT, int NA, bool SM, int NWARP>
+__global__ void __launch_bounds__(32 * NWARP, 32 / NWARP)
+rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
+                    const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
+                    const CellT *__restrict__ init, int32_t *tsteps, int n_steps, uint64_t seed,
+                    const uint8_t *__restrict__ actions, CellT *obs_traj, int32_t *rew_traj,
+                    uint8_t *done_traj, int32_t *rew_sum, uint32_t *status)
+{
+    constexpr int T = 32 * NWARP;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const MemoLayout L = memo_layout(cf, SM);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, env = blockIdx.x;
+    const int C = cf.C, NW = cf.NW, NWP = cf.NWP, HW = cf.HW;
+    const int nbytes = HW * (int)sizeof(CellT);
+    MemoSmem S;
+    S.planes = reinterpret_cast<uint2 *>(smem + L.planes);
+    S.setp = reinterpret_cast<uint32_t *>(smem + L.setp);
+    S.clrp = reinterpret_cast<uint32_t *>(smem + L.clrp);
+    S.basep = reinterpret_cast<uint32_t *>(smem + L.basep);
+    S.vm = reinterpret_cast<uint32_t *>(smem + L.vm);
+    S.masks = reinterpret_cast<uint32_t *>(smem + L.masks);
+    S.cells = reinterpret_cast<uint32_t *>(smem + L.cells);
+    S.red = reinterpret_cast<int *>(smem + L.red);
+    uint4 *hdr = reinterpret_cast<uint4 *>(smem + L.hdr);
+    uint2 *lead = reinterpret_cast<uint2 *>(smem + L.lead);
+    S.hdr = hdr;
+    S.lead = lead;
+    const int table = cf.rules_per_env ? env : 0;
+    const uint32_t *tab_g = arena + tab_off[table];
+    const uint32_t *tab = SM ? reinterpret_cast<const uint32_t *>(smem + L.rules) : tab_g;
+
+    // ---- stage
+    for (int i = tid; i < kShapes * NW; i += T)
+        S.vm[i] = __ldg(vm_g + i);
+    for (int i = tid; i < 3 * NW; i += T)
+        S.masks[i] = __ldg(masks_g + i);
+    if (SM) {
+        const uint32_t n = tab_off[table + 1] - tab_off[table];
+        for (uint32_t i = tid; i < n / 4; i += T)
+            reinterpret_cast<uint4 *>(smem + L.rules)[i] = __ldg(reinterpret_cast<const uint4 *>(tab_g) + i);
+    }
+    for (int i = tid; i < 2 * cf.R; i += T)  // rule headers: words 4 + 8r .. 4 + 8r + 7 of the table
+        hdr[i] = __ldg(reinterpret_cast<const uint4 *>(tab_g + 4) + i);
+    for (int i = tid; i < (C + 2) * NWP; i += T)
+        S.planes[i] = make_uint2(0u, 0u);
+    const uint32_t n_terms = __ldg(tab_g + 1);
+    {
+        const uint2 *terms = reinterpret_cast<const uint2 *>(tab_g + table_terms_word(cf.R));
+        const uint2 pass = make_uint2((uint32_t)(C + 1) * NWP * 8, kTermAbsent);
+        for (int i = tid; i < cf.R * 4 * kMemoLead; i += T) {  // [rule][rotation][term]
+            const int r = i / (4 * kMemoLead), g = (i / kMemoLead) & 3, j = i & (kMemoLead - 1);
+            const uint32_t nt = __ldg(tab_g + 4 + 8 * r) + __ldg(tab_g + 5 + 8 * r);
+            const uint32_t first = __ldg(tab_g + 8 + 8 * r);
+            lead[i] = (uint32_t)j < nt ? __ldg(terms + (size_t)(first + j) * 4 + g) : pass;
+        }
+    }
+    __syncthreads();  // the zeroed planes
+    {
+        // the boards into planes: warp w takes the 32-cell groups w, w + NWARP, ...
+        const CellT *src = cur + (size_t)env * HW, *isrc = init + (size_t)env * HW;
+        for (int base = 32 * warp; base < HW; base += T) {
+            const int p = base + lane;
+            const uint32_t x = p < HW ? (uint32_t)src[p] : 0u;
+            const uint32_t xi = p < HW ? (uint32_t)isrc[p] : 0u;
+            const int w = base >> 5;
+            for (int c = 0; c < C; ++c) {
+                const uint32_t bits = __ballot_sync(0xffffffffu, (x >> c) & 1u);
+                const uint32_t ibits = __ballot_sync(0xffffffffu, (xi >> c) & 1u);
+                if (lane == 0) {
+                    put_word(S.planes, NWP, c, w, bits);
+                    S.basep[c * NW + w] = ibits;
+                }
+            }
+        }
+    }
+    __syncthreads();
+
+    uint32_t v[4 * NA];  // this lane's 16-byte units of the board's canonical bytes
+    memo_cells<CellT, NA, NWARP>(cf, S.planes, S.cells, v);
+    // Outcomes remembered for the current board: bit a of `known` when the step
+    // with action a has been evaluated on it (it leaves the board unchanged),
+    // bit a of `goal` when a goal tile is left after it; lane a holds its reward.
+    uint32_t known = 0, goal = 0;
+    int rew_lane = 0;
+    int t = tsteps[env];
+    int sum = 0, warn = 0;
+    const int obs_mode = obs_traj ? memo_store_mode(obs_traj, nbytes) : 0;
+    const size_t step_stride = (size_t)cf.B * nbytes;  // bytes from one step's boards to the next's
+    unsigned char *const obs_env = obs_traj ? reinterpret_cast<unsigned char *>(obs_traj) + (size_t)env * nbytes
+                                            : nullptr;
+
+    for (int b0 = 0; b0 < n_steps; b0 += 32) {
+        const int lim = min(32, n_steps - b0);
+        const int a_l = lane < lim ? action_at(actions, seed, env, b0 + lane, &warn) : 0;
+        int l0 = 0;
+        while (l0 < lim) {
+            // lane l takes step b0 + l as if no step of this run before it
+            // changed the board, reset the environment or was not yet known
+            const bool act = lane >= l0 && lane < lim;
+            const bool kn_l = (known >> a_l) & 1u;
+            const int r_l = __shfl_sync(0xffffffffu, rew_lane, a_l);
+            const bool goal_l = (goal >> a_l) & 1u;
+            const int t_l = t + (lane - l0) + 1;
+            const bool done_l = !goal_l || (cf.max_steps > 0 && t_l >= cf.max_steps);
+            const uint32_t ev = __ballot_sync(0xffffffffu, act && (!kn_l || (done_l && cf.auto_reset)));
+            const int e = ev ? __ffs(ev) - 1 : lim;  // the first step that is not a plain repeat
+            if (warp == 0 && act && lane < e) {  // steps that repeat the board
+                sum += r_l;
+                if (rew_traj)
+                    rew_traj[(size_t)(b0 + lane) * cf.B + env] = r_l;
+                if (done_traj)
+                    done_traj[(size_t)(b0 + lane) * cf.B + env] = (uint8_t)done_l;
+            }
+            if (obs_traj) {  // the warps take turns
+                unsigned char *o = obs_env + (size_t)(b0 + l0 + warp) * step_stride;
+                for (int l = l0 + warp; l < e; l += NWARP, o += NWARP * step_stride)
+                    memo_store<NA>(o, v, nbytes, obs_mode);
+            }
+            t += e - l0;
+            if (e >= lim)
+                break;
+
+            // ---- step b0 + e (every warp)
+            const int a = __shfl_sync(0xffffffffu, a_l, e);
+            int r, done, changed;
+            if (!((known >> a) & 1u)) {
+                const int2 o = memo_step_eval<NA, SM, NWARP>(cf, tab, n_terms, S, a);
+                if (!(o.y & 1)) {  // the board stays: remember the outcome, take the step again
+                    known |= 1u << a;
+                    if (o.y & 2)
+                        goal |= 1u << a;
+                    if (lane == a)
+                        rew_lane = o.x;
+                    l0 = e;
+                    continue;
+                }
+                r = o.x;
+                t += 1;
+                done = !(o.y & 2) || (cf.max_steps > 0 && t >= cf.max_steps);
+                if (done && cf.auto_reset) {
+                    changed = memo_restore<NWARP>(cf, S.planes, S.basep);
+                    t = 0;
+                } else {
+                    memo_apply<NWARP>(cf, S.planes, S.setp);
+                    changed = 1;
+                }
+            } else {  // a known step that ends in an auto-reset
+                r = __shfl_sync(0xffffffffu, r_l, e);
+                done = 1;
+                changed = memo_restore<NWARP>(cf, S.planes, S.basep);
+                t = 0;
+            }
+            if (warp == 0 && lane == e) {
+                sum += r;
+                if (rew_traj)
+                    rew_traj[(size_t)(b0 + e) * cf.B + env] = r;
+                if (done_traj)
+                    done_traj[(size_t)(b0 + e) * cf.B + env] = (uint8_t)done;
+            }
+            if (changed) {
+                known = goal = 0;
+                memo_cells<CellT, NA, NWARP>(cf, S.planes, S.cells, v);
+            }
+            if (obs_traj && warp == (e % NWARP))
+                memo_store<NA>(obs_env + (size_t)(b0 + e) * step_stride, v, nbytes, obs_mode);
+            l0 = e + 1;
+        }
+    }
+    if (warp == 0) {
+        memo_store<NA>(reinterpret_cast<unsigned char *>(cur) + (size_t)env * nbytes, v, nbytes,
+                       memo_store_mode(cur, nbytes));
+        sum = __reduce_add_sync(0xffffffffu, sum);
+        warn = __any_sync(0xffffffffu, warn);
+        if (lane == 0) {
+            tsteps[env] = t;
+            if (rew_sum)
+                rew_sum[env] = sum;
+            if (warn)
+                atomicOr(status + 1, kWarnAction);
+        }
+    }
+}
+
+}  // namespace av
+
+// ---------------------------------------------------------------- launchers
+// Compiled once per cell type (AV_MEMO_CELL) by k_memo_u8.cu / k_memo_u16.cu.
+#ifdef AV_MEMO_CELL
+namespace av {
+namespace AV_MEMO_NS {
+
+template <typename CellT, int NA, bool SM, int NWARP>
+void memo_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+            const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
+            const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
+            uint32_t *status, cudaStream_t st)
+{
+    const size_t sm = memo_layout(cf, SM).total;
+    rollout_memo_kernel<CellT, NA, SM, NWARP><<<cf.B, 32 * NWARP, sm, st>>>(
+        cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
+        (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
+}
+
+template <typename CellT, int NA, bool SM>
+void memo_w(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+            const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
+            const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
+            uint32_t *status, cudaStream_t st)
+{
+#define AV_MEMO(NWARP)                                                                                     \
+    memo_t<CellT, NA, SM, NWARP>(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj, \
+                                 rew_traj, done_traj, rew_sum, status, st)
+    switch (memo_warps(cf)) {
+    case 1: AV_MEMO(1); break;
+    case 2: AV_MEMO(2); break;
+    default: AV_MEMO(4); break;
+    }
+#undef AV_MEMO
+}
+
+}  // namespace AV_MEMO_NS
+
+cudaError_t AV_MEMO_CONFIGURE()
+{
+    cudaError_t e = cudaSuccess;
+    auto set = [&](const void *fn) {
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmemLimit);
+    };
+#define AV_SETM(NA, SM) \
+    set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 1>); \
+    set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 2>); \
+    set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 4>);
+    AV_SETM(1, true)
+    AV_SETM(1, false)
+    AV_SETM(2, true)
+    AV_SETM(2, false)
+#undef AV_SETM
+    return e;
+}
+
+void AV_MEMO_LAUNCH(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+                    const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
+                    const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj,
+                    int32_t *rew_sum, uint32_t *status, cudaStream_t st)
+{
+#define AV_MEMO(NA, SM)                                                                                  \
+    AV_MEMO_NS::memo_w<AV_MEMO_CELL, NA, SM>(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed,   \
+                                             actions, obs_traj, rew_traj, done_traj, rew_sum, status, st)
+    const bool staged = memo_staged(cf);
+    if (cf.NA == 1) {
+        if (staged) AV_MEMO(1, true);
+        else AV_MEMO(1, false);
+    } else {
+        if (staged) AV_MEMO(2, true);
+        else AV_MEMO(2, false);
+    }
+#undef AV_MEMO
+}
+
+}  // namespace av
+#endif

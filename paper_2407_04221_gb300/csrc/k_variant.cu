@@ -642,11 +642,8 @@ cudaError_t configure_variant()
     return e;
 }
 
-// One warp per environment where the standard step would run the one-warp
-// rollout (small boards, few rules, rule sets not flagged busy, or
-// AV_KERNEL_PATH=warp); else one CTA per environment.
-static bool use_variant_warp(const DevConfig &cf) { return use_env_warp_rollout(cf); }
-
+// One warp per environment for small boards with few rules whose rule set is
+// not flagged busy (use_variant_warp), else one CTA per environment.
 void launch_rollout_variant(const DevConfig &cf, const VariantParams &vp, const uint32_t *arena,
                             const uint32_t *tab_off, const uint32_t *vm, const uint32_t *masks, void *cur,
                             const void *init, int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions,

@@ -67,9 +67,11 @@ struct DevConfig {
     int ch_player, ch_goal, ch_empty, ch_wall, border_wall, cum_per_env;
     int cell_bytes;
     int rule_words;  // largest rule table (words) when tables are staged in shared memory, else 0
-    int path;        // 0: choose; 1: block kernels; 2: fast rollout; 3: one warp per env
+    int path;        // 0: choose; 1: block kernels; 2: fast rollout; 3: one warp per env; 4: memoising rollout
     int busy;        // rules expected to pass their register terms on most steps (host estimate)
     int fast_warps;  // fast rollout: warps per environment (4, or 8 when set to 8)
+    int memo_stage;  // memo rollout: 0 the library decides, 1 rule tables in shared memory, 2 not
+    int memo_warps;  // memo rollout: warps per environment (0: the default)
 };
 
 // Rule-table helpers shared by host (compiler) and device (reader).
@@ -2479,18 +2481,23 @@ inline int anchor_slots(int NW)
 }
 
 // Paths: cf.path 0 = choose, 1 = block per env, 2 = fast rollout (several warps
-// per env), 3 = one warp per env.
-// Rollouts: one warp per environment for boards of at most 16 plane words and
-// at most 16 rules, else the fast kernel for <= 64 rules, else (or when forced)
-// the block kernel; rule sets flagged busy take the block kernel.  Expansion: one warp per parent for boards of at most 16
-// plane words unless the block path is forced.
-inline bool use_env_warp_rollout(const DevConfig &cf)
-{
-    return cf.NA <= 2 && cf.R <= 16 && ((cf.path == 0 && !cf.busy) || cf.path == 3);
-}
+// per env), 3 = one warp per env, 4 = the memoising rollout.
+// Rollouts: the memoising rollout (k_memo_impl.cuh) for boards of at most 16
+// plane words, any rule count; else (or when forced) the block kernel.  The
+// one-warp kernel (at most 16 rules) and the fast kernel (at most 64 rules)
+// run when AV_KERNEL_PATH asks for them.  Expansion: one warp per parent for
+// boards of at most 16 plane words unless the block path is forced.
+inline bool use_memo_rollout(const DevConfig &cf) { return cf.NA <= 2 && (cf.path == 0 || cf.path == 4); }
+inline bool use_env_warp_rollout(const DevConfig &cf) { return cf.NA <= 2 && cf.R <= 16 && cf.path == 3; }
 inline bool use_fast_rollout(const DevConfig &cf)
 {
-    return cf.NA <= 2 && cf.R <= 64 && ((cf.path == 0 && !cf.busy) || cf.path == 2 || cf.path == 3);
+    return cf.NA <= 2 && cf.R <= 64 && (cf.path == 2 || cf.path == 3);
+}
+// Variant semantics: one warp per environment for small boards with at most
+// 16 rules unless the rule set is flagged busy or another path is forced.
+inline bool use_variant_warp(const DevConfig &cf)
+{
+    return cf.NA <= 2 && cf.R <= 16 && ((cf.path == 0 && !cf.busy) || cf.path == 3 || cf.path == 4);
 }
 inline bool use_warp_expand(const DevConfig &cf) { return cf.NA <= 2 && cf.path != 1; }
 

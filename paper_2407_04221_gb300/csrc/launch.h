@@ -19,6 +19,8 @@ cudaError_t configure_block();
 cudaError_t configure_expand();
 cudaError_t configure_search();
 cudaError_t configure_observe();
+cudaError_t configure_memo_u8();
+cudaError_t configure_memo_u16();
 
 void launch_rollout_fast_u8(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
                             const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
@@ -36,6 +38,16 @@ void launch_rollout_warp_u8(const DevConfig &cf, const uint32_t *arena, const ui
                             int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
                             cudaStream_t st);
 void launch_rollout_warp_u16(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
+                             const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
+                             int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
+                             int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                             cudaStream_t st);
+void launch_rollout_memo_u8(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
+                            const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
+                            int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
+                            int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
+                            cudaStream_t st);
+void launch_rollout_memo_u16(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
                              const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
                              int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
                              int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
@@ -113,6 +125,8 @@ inline cudaError_t configure_kernels()
     if (e == cudaSuccess) e = configure_expand();
     if (e == cudaSuccess) e = configure_search();
     if (e == cudaSuccess) e = configure_observe();
+    if (e == cudaSuccess) e = configure_memo_u8();
+    if (e == cudaSuccess) e = configure_memo_u16();
     if (e == cudaSuccess) e = configure_variant();
     if (e == cudaSuccess) e = configure_band();
     return e;
@@ -124,7 +138,13 @@ inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uin
                            int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
                            cudaStream_t st)
 {
-    if (use_env_warp_rollout(cf) && cf.cell_bytes == 1)
+    if (use_memo_rollout(cf) && cf.cell_bytes == 1)
+        launch_rollout_memo_u8(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
+                               rew_traj, done_traj, rew_sum, status, st);
+    else if (use_memo_rollout(cf))
+        launch_rollout_memo_u16(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
+                                rew_traj, done_traj, rew_sum, status, st);
+    else if (use_env_warp_rollout(cf) && cf.cell_bytes == 1)
         launch_rollout_warp_u8(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
                                rew_traj, done_traj, rew_sum, status, st);
     else if (use_env_warp_rollout(cf))

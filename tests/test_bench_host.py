@@ -113,3 +113,50 @@ def test_committed_profiles_name_their_kernel_sources():
         text = open(path).read()
         if "dram_bytes_per_launch:" in text:
             assert re.search(r"kernel_source_sha256:\s*[0-9a-f]{16}", text), path
+
+
+def test_row_basis_ops_by_hand():
+    """One op per (rule rotation, input or output entry, valid anchor row)."""
+    wl = wk.Workload(0, "t", 1, 4, 6, 2, 2, ((1, 1),), 0.1, 0.1, 0.1, 0.1, 0, 0)
+    rules = wk.empty_rules(1, 2)
+    rules["h"], rules["w"] = [[1, 2]], [[1, 3]]
+    rules["present"][0, 0, 0] = 0b11      # 2 input entries
+    rules["set"][0, 0, 0] = 0b01          # 1 output entry
+    rules["absent"][0, 1, 5] = 0b10       # 1 input entry
+    rules["clear"][0, 1, 0] = 0b11        # 2 output entries
+    # rule 0, 1x1: 4 rotations x 4 rows x 3 entries; rule 1, 2x3: rotations 0, 2
+    # have 4 - 2 + 1 = 3 rows, rotations 1, 3 (3x2) have 4 - 3 + 1 = 2 rows, x 3 entries
+    assert bench.row_basis_ops(wl, rules) == 4 * 4 * 3 + (2 * 3 + 2 * 2) * 3
+
+
+def test_trajectory_bytes_and_default_workload():
+    wl3 = wk.WORKLOADS[3]
+    assert bench.traj_bytes_per_env_step(wl3) == 16 * 16 * 2 + 4 + 1
+    import argparse  # noqa: F401
+    # the default benchmark line is the largest single-GPU workload (config 3)
+    src = open(os.path.join(ROOT, "bench.py")).read()
+    assert '"--config", type=int, default=3' in src
+
+
+def test_search_workload_names_its_base_game_rules():
+    d = bench.config_dict(wk.WORKLOADS[4])
+    assert "move and eat rules" in d["workload"]
+    assert "far exceed L2" in bench.config_dict(wk.WORKLOADS[3])["l2"]
+
+
+def test_single_step_actions_match_the_rollout_draw():
+    """The single-step benchmark's actions are the fused rollout's on-device
+    draws (SplitMix64 counter, stream 4), recomputed independently here."""
+    a = wk.actions(7, 3, 4)
+    M = (1 << 64) - 1
+
+    def mix(z):
+        z = ((z ^ (z >> 30)) * 0xbf58476d1ce4e5b9) & M
+        z = ((z ^ (z >> 27)) * 0x94d049bb133111eb) & M
+        return z ^ (z >> 31)
+    for s in range(4):
+        for e in range(3):
+            z = mix((7 + 0x9E3779B97F4A7C15 * 5) & M)
+            z = mix(z ^ e)
+            d = mix(z ^ s)
+            assert a[s, e] == ((d >> 32) * 5) >> 32

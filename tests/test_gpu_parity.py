@@ -214,9 +214,9 @@ def test_dense_matches_stress_apply():
 
 
 # ------------------------------------------------- both kernel paths
-_PATH_IDS = {"block": 1, "fast": 2, "fast8": 2, "warp": 3}
+_PATH_IDS = {"block": 1, "fast": 2, "fast8": 2, "warp": 3, "memo": 6}
 
-@pytest.mark.parametrize("path", ["block", "fast", "fast8", "warp"])
+@pytest.mark.parametrize("path", ["block", "fast", "fast8", "warp", "memo"])
 @pytest.mark.parametrize("key,batch,steps", [(1, 3, 60), (2, 9, 70), (3, 7, 230), (4, 4, 30)])
 def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
     import paper_2407_04221_gb300 as av
@@ -238,7 +238,7 @@ def test_both_kernel_paths_rollout(monkeypatch, path, key, batch, steps):
     env.close()
 
 
-@pytest.mark.parametrize("path", ["block", "fast", "fast8", "warp"])
+@pytest.mark.parametrize("path", ["block", "fast", "fast8", "warp", "memo"])
 @pytest.mark.parametrize("H,W,C,shapes,R", [
     (1, 1, 1, ((1, 1),), 2),
     (7, 9, 3, ((3, 3), (5, 5), (1, 4)), 4),
@@ -275,7 +275,7 @@ def test_both_kernel_paths_edges(monkeypatch, path, H, W, C, shapes, R):
 
 
 # ------------------------------------- launch lengths around the action ring
-@pytest.mark.parametrize("path", ["block", "fast", "warp"])
+@pytest.mark.parametrize("path", ["block", "fast", "warp", "memo"])
 def test_launch_lengths_and_continuation(monkeypatch, path):
     """Rollouts of 0 and 1 steps, lengths around the 128-step refill of the
     pre-drawn actions, and launches that continue one another, each compared

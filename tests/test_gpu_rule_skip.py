@@ -94,7 +94,7 @@ def _check(env, shape, variant, steps=200, action_seed=11):
 
 
 @pytest.mark.parametrize("shape", list(SHAPES))
-@pytest.mark.parametrize("path", ["warp", "fast", "block", "default"])
+@pytest.mark.parametrize("path", ["warp", "fast", "block", "memo", "default"])
 def test_standard(path, shape, monkeypatch):
     import paper_2407_04221_gb300 as av
     if path != "default":
@@ -103,6 +103,8 @@ def test_standard(path, shape, monkeypatch):
     env = av.Env(_fields(H, W, 3 * copies), _rules(copies))
     if path == "warp":
         assert av.av_rollout_path(env.h) == av.AV_PATH_WARP
+    if path == "memo":
+        assert av.av_rollout_path(env.h) == av.AV_PATH_MEMO
     _check(env, shape, None)
     env.sync()
     env.close()

@@ -272,6 +272,15 @@ def make_init_cum(wl: Workload, seed: int) -> np.ndarray:
     return cum
 
 
+def actions(seed: int, batch: int, n_steps: int) -> np.ndarray:
+    """Actions [n_steps][batch] uint8 in 0..4 for step-by-step runs: step s of
+    env e takes uniform_int(draw(seed, 4, e, 0, s), 5), the same action a fused
+    rollout with action seed `seed` draws on the device."""
+    e = np.arange(batch, dtype=np.uint64)[None, :]
+    st = np.arange(n_steps, dtype=np.uint64)[:, None]
+    return uniform_int(draw(seed, 4, e, np.uint64(0), st), 5).astype(np.uint8)
+
+
 def config_fields(wl: Workload) -> dict:
     """Scalar fields of the library's / oracle's configuration structs."""
     def role(ch):
