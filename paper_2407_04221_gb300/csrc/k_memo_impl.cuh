@@ -36,13 +36,18 @@ constexpr int kMemoLead = 4;  // leading terms of each rule tested for all rules
 // Shared memory of one environment (one CTA): the valid-anchor and column
 // masks; tile planes 0..C-1, the force of the action being evaluated (plane
 // C) and an all-zero plane C+1 (padding terms read it as absent and pass),
-// doubled; SET and CLEAR planes (SET becomes the flip planes of the evaluated
-// step); the initial map's planes (flat); per rule its two header words
-// (uint4 each) and its first kMemoLead terms in each rotation; the board's
-// canonical bytes; per-warp reductions; the whole rule table when staged.
+// doubled; per warp a SET and a CLEAR plane set (each warp ORs the outputs of
+// its own rules there); for each of two board slots (the current board and
+// the one before it) the flip planes of each action's step, the board's planes
+// (flat) and its canonical bytes; the initial map's planes (flat); per rule its
+// two header words (uint4 each) and its first kMemoLead terms in each rotation;
+// per-warp reductions; the whole rule table when staged.
 struct MemoLayout {
-    size_t vm, masks, planes, setp, clrp, basep, hdr, lead, cells, red, rules, total;
+    size_t vm, masks, planes, acc, flip, bplanes, basep, hdr, lead, cells, red, rules, total;
 };
+
+// Warps per environment (CTA): AV_MEMO_WARPS=1|2|4, read by av_create, else 2.
+__host__ __device__ inline int memo_warps(const DevConfig &cf) { return cf.memo_warps == 1 || cf.memo_warps == 4 ? cf.memo_warps : 2; }
 
 __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool staged)
 {
@@ -51,20 +56,18 @@ __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool stag
     L.vm = 0;
     L.masks = align16((size_t)kShapes * cf.NW * 4);
     L.planes = align16(L.masks + (size_t)3 * cf.NW * 4);
-    L.setp = align16(L.planes + (size_t)(cf.C + 2) * cf.NWP * 8);
-    L.clrp = align16(L.setp + pw);
-    L.basep = align16(L.clrp + pw);
+    L.acc = align16(L.planes + (size_t)(cf.C + 2) * cf.NWP * 8);
+    L.flip = align16(L.acc + 2 * (size_t)memo_warps(cf) * pw);
+    L.bplanes = align16(L.flip + 10 * pw);
+    L.basep = align16(L.bplanes + 2 * pw);
     L.hdr = align16(L.basep + pw);
     L.lead = align16(L.hdr + (size_t)cf.R * 32);
     L.cells = align16(L.lead + (size_t)cf.R * 4 * kMemoLead * 8);
-    L.red = align16(L.cells + (size_t)cf.HW * cf.cell_bytes);
+    L.red = align16(L.cells + 2 * align16((size_t)cf.HW * cf.cell_bytes));
     L.rules = align16(L.red + 16 * 4);
     L.total = align16(L.rules + (staged ? (size_t)cf.rule_words * 4 : 0));
     return L;
 }
-
-// Warps per environment (CTA): AV_MEMO_WARPS=1|2|4, read by av_create, else 2.
-inline int memo_warps(const DevConfig &cf) { return cf.memo_warps == 1 || cf.memo_warps == 4 ? cf.memo_warps : 2; }
 
 // Whether the whole rule table is copied into shared memory: when the
 // environment's region with it still lets as many environments share an SM
@@ -125,8 +128,12 @@ __host__ __device__ inline int memo_store_mode(const void *p, int nbytes)
 // Shared memory of one environment, as pointers.
 struct MemoSmem {
     uint2 *planes;
-    uint32_t *setp, *clrp, *basep, *vm, *masks, *cells;
-    int *red;           // [w] reward of warp w's rules; [8] a bit flips; [9] a goal tile is left
+    uint32_t *acc;   // [warp][SET, CLEAR][C * NW]
+    uint32_t *flip;     // [slot][action][C * NW]: the bits each remembered step flips
+    uint32_t *bplanes;  // [slot][C * NW]: each slot's board
+    uint32_t *basep, *vm, *masks, *cells;
+    int *red;           // [w] reward of warp w's rules; [8] a bit flips; [9] a goal tile is left;
+                        // [10], [11] rules 0-31 / 32-63 that pass their leading terms
     const uint4 *hdr;   // [R][2]: (n_present, n_absent, n_out, reward), (first term, first output, shapes, 0)
     const uint2 *lead;  // [R][4 rotations][kMemoLead] term descriptors
 };
@@ -157,27 +164,81 @@ __device__ __forceinline__ void memo_lead(const DevConfig &cf, const MemoSmem &S
     }
 }
 
+// The outputs of one rule (n_out entries at `op`, this lane's rotation) at
+// the live anchors m of its four rotations, ORed into this warp's SET / CLEAR
+// planes without atomics.  Output entry at window offset s = 32 d + sh moves
+// the anchors of word j to word j + d (shifted left by sh) and j + d + 1; so
+// the owner of word W takes (M[W - d] << sh) | (M[W - d - 1] >> (32 - sh)),
+// fetching its rotation's match words by shuffles (word j of a rotation is lane
+// (j & 7) of its quarter, anchor-word slot j >> 3).  The four rotations' words
+// are ORed by two xor-shuffles, and the lanes of quarter 0 write each word
+// (one lane per word, a plain read-modify-write in the warp's own planes).
+template <int NA, bool SM>
+__device__ __forceinline__ void memo_write(const DevConfig &cf, const uint4 *op, uint32_t n_out,
+                                           const uint32_t (&m)[NA], uint32_t *wset, uint32_t *wclr)
+{
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    for (uint32_t o = 0; o < n_out; ++o) {
+        const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
+        const int d = (int)ov.x;
+        const uint32_t sh = ov.y;
+        uint32_t cw[NA];
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            const int a = q + 8 * u - d, b = a - 1;  // source words of the low and high parts
+            uint32_t xa = 0, xb = 0;
+#pragma unroll
+            for (int v = 0; v < NA; ++v) {
+                const uint32_t ya = __shfl_sync(0xffffffffu, m[v], (g << 3) | (a & 7));
+                const uint32_t yb = __shfl_sync(0xffffffffu, m[v], (g << 3) | (b & 7));
+                if (a >= 0 && (a >> 3) == v)
+                    xa = ya;
+                if (b >= 0 && (b >> 3) == v)
+                    xb = yb;
+            }
+            uint32_t c = (xa << sh) | (sh ? (xb >> (32u - sh)) : 0u);
+            c |= __shfl_xor_sync(0xffffffffu, c, 8);
+            c |= __shfl_xor_sync(0xffffffffu, c, 16);
+            cw[u] = c;
+        }
+        if (g == 0) {
+#pragma unroll
+            for (int u = 0; u < NA; ++u) {
+                const int W = q + 8 * u;
+                if (W >= cf.NW || !cw[u])
+                    continue;
+                for (uint32_t ch = ov.z; ch; ch &= ch - 1)
+                    wset[(__ffs(ch) - 1) * cf.NW + W] |= cw[u];
+                for (uint32_t ch = ov.w; ch; ch &= ch - 1)
+                    wclr[(__ffs(ch) - 1) * cf.NW + W] |= cw[u];
+            }
+        }
+        __syncwarp();
+    }
+}
+
 // One step of the board in S.planes with action `a`, by all NWARP warps of the
-// CTA: every rule in its four rotations as in the step-by-step kernels (warp w
-// takes rules w, w + NWARP, ...): the force plane of `a`, the leading terms of
-// the warp's rules, the remaining terms of those that pass them (four per
-// vote), the outputs of live matches ORed into SET / CLEAR; then the flip
-// planes (SET bits on clear cells, CLEAR bits on set cells) in place of
-// S.setp.  `n_terms` is the table's term count (its word 1).  Returns
+// CTA: every rule in its four rotations as in the step-by-step kernels: the
+// force plane of `a`, the leading terms of every rule (warp w takes rules w,
+// w + NWARP, ...), then the rules that pass them dealt out among the warps
+// afresh, so that a few live rules do not fall to one warp: their remaining
+// terms (four per
+// vote), the outputs of live matches ORed into the warp's own SET / CLEAR
+// planes (memo_write); then the flip planes flip_out (SET bits on clear cells,
+// CLEAR bits on set cells, over every warp's planes).  `n_terms` is the
+// table's term count (its word 1).  Returns
 // (reward, bit 0: the step changes the board, bit 1: a goal tile is left
 // after it, always without a goal channel), the same in every thread.  Not
 // inlined: it runs once per board and action.
 template <int NA, bool SM, int NWARP>
-static __device__ __noinline__ int2 memo_step_eval(DevConfig cf, const uint32_t *tab, uint32_t n_terms, MemoSmem S,
-                                                   int a)
+static __device__ __forceinline__ int2 memo_step_eval(DevConfig cf, const uint32_t *tab, uint32_t n_terms, MemoSmem S,
+                                                       int a, uint32_t *flip_out)
 {
     constexpr int T = 32 * NWARP;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 3, q = lane & 7;
     const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
-    for (int i = tid; i < cnw; i += T) {
-        S.setp[i] = 0u;
-        S.clrp[i] = 0u;
-    }
+    for (int i = tid; i < 2 * NWARP * cnw; i += T)
+        S.acc[i] = 0u;
     if (tid < 16)
         S.red[tid] = 0;
     if (warp == NWARP - 1)
@@ -202,6 +263,25 @@ static __device__ __noinline__ int2 memo_step_eval(DevConfig cf, const uint32_t 
     }
     alive0 = __reduce_or_sync(0xffffffffu, alive0);
     alive1 = cf.R > 32 ? __reduce_or_sync(0xffffffffu, alive1) : 0u;
+    if (NWARP > 1) {
+        // the rules that passed, dealt out afresh: the k-th of them to warp k mod NWARP
+        if (lane == 0) {
+            if (alive0)
+                atomicOr(reinterpret_cast<unsigned int *>(S.red) + 10, alive0);
+            if (alive1)
+                atomicOr(reinterpret_cast<unsigned int *>(S.red) + 11, alive1);
+        }
+        __syncthreads();
+        const uint32_t all0 = (uint32_t)S.red[10], all1 = (uint32_t)S.red[11];
+        alive0 = alive1 = 0;
+        int k = 0;
+        for (uint32_t x = all0; x; x &= x - 1, ++k)
+            if (k % NWARP == warp)
+                alive0 |= x & (0u - x);
+        for (uint32_t x = all1; x; x &= x - 1, ++k)
+            if (k % NWARP == warp)
+                alive1 |= x & (0u - x);
+    }
     const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
     const uint4 *outs = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, n_terms));
     const uint32_t pass_x = (uint32_t)(cf.C + 1) * NWP * 8;  // a term on the zero plane, read as absent
@@ -242,24 +322,11 @@ static __device__ __noinline__ int2 memo_step_eval(DevConfig cf, const uint32_t 
 #pragma unroll
             for (int u = 0; u < NA; ++u)
                 cnt += __popc(m[u]);
-            if (cnt) {  // this lane's live anchors pay and write
+            if (__any_sync(0xffffffffu, cnt != 0u)) {  // the rule matched: it pays and writes
                 rew += (int)h0.w * (int)cnt;
-                const uint4 *op = outs + (size_t)h1.y * 4 + g;
-                for (uint32_t o = 0; o < h0.z; ++o) {
-                    const uint4 ov = SM ? op[4 * o] : __ldg(op + 4 * o);
-#pragma unroll
-                    for (int u = 0; u < NA; ++u) {
-                        if (!m[u])
-                            continue;
-                        const int w0 = q + 8 * u + (int)ov.x;
-                        const uint32_t lo = m[u] << ov.y;
-                        const uint32_t hi = ov.y ? (m[u] >> (32u - ov.y)) : 0u;
-                        scatter_bits(S.setp, ov.z, NW, w0, lo, hi);
-                        scatter_bits(S.clrp, ov.w, NW, w0, lo, hi);
-                    }
-                }
+                memo_write<NA, SM>(cf, outs + (size_t)h1.y * 4 + g, h0.z, m, S.acc + (size_t)warp * 2 * cnw,
+                                   S.acc + (size_t)warp * 2 * cnw + cnw);
             }
-            __syncwarp();
         }
     }
     rew = __reduce_add_sync(0xffffffffu, rew);
@@ -267,11 +334,20 @@ static __device__ __noinline__ int2 memo_step_eval(DevConfig cf, const uint32_t 
         S.red[warp] = rew;
     __syncthreads();  // every warp's SET / CLEAR bits and reward
     uint32_t any = 0, goal = 0;
-    for (int i = tid; i < cnw; i += T) {
-        const int c = i / NW, w = i - c * NW;
+    for (int i = tid, c = tid / NW, w = tid - (tid / NW) * NW; i < cnw; i += T, c += T / NW, w += T % NW) {
+        if (w >= NW) {  // (c, w) of i = c * NW + w, stepped by T = (T / NW) * NW + T % NW
+            w -= NW;
+            ++c;
+        }
+        uint32_t st = 0, cl = 0;
+#pragma unroll
+        for (int k = 0; k < NWARP; ++k) {
+            st |= S.acc[2 * k * cnw + i];
+            cl |= S.acc[(2 * k + 1) * cnw + i];
+        }
         const uint32_t d = S.planes[c * NWP + w].x;
-        const uint32_t f = (d & S.clrp[i]) | (~d & S.setp[i]);  // a bit changes where a match asks for it
-        S.setp[i] = f;
+        const uint32_t f = (d & cl) | (~d & st);  // a bit changes where a match asks for it
+        flip_out[i] = f;
         any |= f;
         if (c == cf.ch_goal)
             goal |= d ^ f;
@@ -294,12 +370,17 @@ static __device__ __noinline__ int2 memo_step_eval(DevConfig cf, const uint32_t 
 
 // The board after its step: planes ^= flip (all warps).
 template <int NWARP>
-static __device__ __noinline__ void memo_apply(DevConfig cf, uint2 *planes, const uint32_t *flip)
+static __device__ __forceinline__ void memo_apply(DevConfig cf, uint2 *planes, const uint32_t *flip)
 {
     const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
-    for (int i = threadIdx.x; i < cnw; i += 32 * NWARP) {
+    constexpr int T = 32 * NWARP;
+    const int tid = threadIdx.x;
+    for (int i = tid, c = tid / NW, w = tid - (tid / NW) * NW; i < cnw; i += T, c += T / NW, w += T % NW) {
+        if (w >= NW) {
+            w -= NW;
+            ++c;
+        }
         const uint32_t f = flip[i];
-        const int c = i / NW, w = i - c * NW;
         if (f)
             put_word(planes, NWP, c, w, planes[c * NWP + w].x ^ f);
     }
@@ -309,19 +390,68 @@ static __device__ __noinline__ void memo_apply(DevConfig cf, uint2 *planes, cons
 // Auto-reset: the initial map's planes back into the tile planes (all warps).
 // Returns whether the board differed from the initial map (every thread).
 template <int NWARP>
-static __device__ __noinline__ int memo_restore(DevConfig cf, uint2 *planes, const uint32_t *basep)
+static __device__ __forceinline__ int memo_restore(DevConfig cf, uint2 *planes, const uint32_t *basep)
 {
     const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
     int diff = 0;
-    for (int i = threadIdx.x; i < cnw; i += 32 * NWARP) {
+    constexpr int T = 32 * NWARP;
+    const int tid = threadIdx.x;
+    for (int i = tid, c = tid / NW, w = tid - (tid / NW) * NW; i < cnw; i += T, c += T / NW, w += T % NW) {
+        if (w >= NW) {
+            w -= NW;
+            ++c;
+        }
         const uint32_t b = basep[i];
-        const int c = i / NW, w = i - c * NW;
         if (planes[c * NWP + w].x != b) {
             diff = 1;
             put_word(planes, NWP, c, w, b);
         }
     }
     return __syncthreads_or(diff);
+}
+
+// The current tile planes (flat) into `bpl` (all warps); returns whether they
+// differed from what `bpl` held (every thread).
+template <int NWARP>
+static __device__ __forceinline__ int memo_switch(const DevConfig &cf, const uint2 *planes, uint32_t *bpl)
+{
+    constexpr int T = 32 * NWARP;
+    const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW, tid = threadIdx.x;
+    int diff = 0;
+    for (int i = tid, c = tid / NW, w = tid - (tid / NW) * NW; i < cnw; i += T, c += T / NW, w += T % NW) {
+        if (w >= NW) {
+            w -= NW;
+            ++c;
+        }
+        const uint32_t x = planes[c * NWP + w].x;
+        diff |= bpl[i] != x;
+        bpl[i] = x;
+    }
+    return __syncthreads_or(diff);
+}
+
+// This lane's 16-byte units of a board's canonical bytes from `cells`.
+template <int NV>
+__device__ __forceinline__ void memo_load_cells(const uint32_t *cells, int n16, uint32_t (&v)[4 * NV])
+{
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+        const int u = lane + 32 * j;
+        const uint4 x = u < n16 ? reinterpret_cast<const uint4 *>(cells)[u] : make_uint4(0u, 0u, 0u, 0u);
+        v[4 * j] = x.x;
+        v[4 * j + 1] = x.y;
+        v[4 * j + 2] = x.z;
+        v[4 * j + 3] = x.w;
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ void swap_vals(T &a, T &b)
+{
+    const T t = a;
+    a = b;
+    b = t;
 }
 
 // The board's canonical bytes into `cells` (shared, a whole number of
@@ -349,16 +479,7 @@ __device__ __forceinline__ void memo_cells(const DevConfig &cf, const uint2 *pla
         cells[k] = x;
     }
     __syncthreads();
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int j = 0; j < NV; ++j) {
-        const int u = lane + 32 * j;
-        const uint4 x = u < n16 ? reinterpret_cast<const uint4 *>(cells)[u] : make_uint4(0u, 0u, 0u, 0u);
-        v[4 * j] = x.x;
-        v[4 * j + 1] = x.y;
-        v[4 * j + 2] = x.z;
-        v[4 * j + 3] = x.w;
-    }
+    memo_load_cells<NV>(cells, n16, v);
 }
 
 // Fused rollout, one CTA of NWARP warps per environment; see the top of this
@@ -376,12 +497,13 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
     extern __shared__ __align__(16) unsigned char smem[];
     const MemoLayout L = memo_layout(cf, SM);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, env = blockIdx.x;
-    const int C = cf.C, NW = cf.NW, NWP = cf.NWP, HW = cf.HW;
+    const int C = cf.C, NW = cf.NW, NWP = cf.NWP, HW = cf.HW, cnw = C * NW;
     const int nbytes = HW * (int)sizeof(CellT);
     MemoSmem S;
     S.planes = reinterpret_cast<uint2 *>(smem + L.planes);
-    S.setp = reinterpret_cast<uint32_t *>(smem + L.setp);
-    S.clrp = reinterpret_cast<uint32_t *>(smem + L.clrp);
+    S.acc = reinterpret_cast<uint32_t *>(smem + L.acc);
+    S.flip = reinterpret_cast<uint32_t *>(smem + L.flip);
+    S.bplanes = reinterpret_cast<uint32_t *>(smem + L.bplanes);
     S.basep = reinterpret_cast<uint32_t *>(smem + L.basep);
     S.vm = reinterpret_cast<uint32_t *>(smem + L.vm);
     S.masks = reinterpret_cast<uint32_t *>(smem + L.masks);
@@ -442,12 +564,21 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
     __syncthreads();
 
     uint32_t v[4 * NA];  // this lane's 16-byte units of the board's canonical bytes
-    memo_cells<CellT, NA, NWARP>(cf, S.planes, S.cells, v);
-    // Outcomes remembered for the current board: bit a of `known` when the step
-    // with action a has been evaluated on it (it leaves the board unchanged),
-    // bit a of `goal` when a goal tile is left after it; lane a holds its reward.
-    uint32_t known = 0, goal = 0;
-    int rew_lane = 0;
+    // Two board slots: the current board (slot cs) and the one before it.  Per
+    // slot: the board's planes (flat, S.bplanes) and canonical bytes (S.cells),
+    // and the outcomes remembered for it, in registers the same in every warp:
+    // bit a of kq[s] when action a leaves the board unchanged, of kc[s] when it
+    // changes it (its flip planes kept in S.flip[s][a]), of gm[s] when a goal
+    // tile is left after it; lane a holds its reward in rw[s].
+    const int n16 = (HW * (int)sizeof(CellT) + 15) / 16;  // 16-byte units of a board
+    // the current slot and the other one (swapped when the board changes)
+    uint32_t *cells_c = S.cells, *cells_o = S.cells + 4 * n16;
+    uint32_t *bpl_c = S.bplanes, *bpl_o = S.bplanes + cnw;
+    uint32_t *flip_c = S.flip, *flip_o = S.flip + 5 * cnw;
+    uint32_t kq = 0u, kc = 0u, gm = 0u, okq = 0u, okc = 0u, ogm = 0u;
+    int rw = 0, orw = 0, valid_other = 0;
+    memo_switch<NWARP>(cf, S.planes, bpl_c);
+    memo_cells<CellT, NA, NWARP>(cf, S.planes, cells_c, v);
     int t = tsteps[env];
     int sum = 0, warn = 0;
     const int obs_mode = obs_traj ? memo_store_mode(obs_traj, nbytes) : 0;
@@ -461,14 +592,15 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
         int l0 = 0;
         while (l0 < lim) {
             // lane l takes step b0 + l as if no step of this run before it
-            // changed the board, reset the environment or was not yet known
+            // changed the board, reset the environment or had no remembered
+            // outcome that leaves the board as it is
             const bool act = lane >= l0 && lane < lim;
-            const bool kn_l = (known >> a_l) & 1u;
-            const int r_l = __shfl_sync(0xffffffffu, rew_lane, a_l);
-            const bool goal_l = (goal >> a_l) & 1u;
+            const bool q_l = (kq >> a_l) & 1u;
+            const int r_l = __shfl_sync(0xffffffffu, rw, a_l);
+            const bool goal_l = (gm >> a_l) & 1u;
             const int t_l = t + (lane - l0) + 1;
             const bool done_l = !goal_l || (cf.max_steps > 0 && t_l >= cf.max_steps);
-            const uint32_t ev = __ballot_sync(0xffffffffu, act && (!kn_l || (done_l && cf.auto_reset)));
+            const uint32_t ev = __ballot_sync(0xffffffffu, act && (!q_l || (done_l && cf.auto_reset)));
             const int e = ev ? __ffs(ev) - 1 : lim;  // the first step that is not a plain repeat
             if (warp == 0 && act && lane < e) {  // steps that repeat the board
                 sum += r_l;
@@ -488,33 +620,43 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
 
             // ---- step b0 + e (every warp)
             const int a = __shfl_sync(0xffffffffu, a_l, e);
-            int r, done, changed;
-            if (!((known >> a) & 1u)) {
-                const int2 o = memo_step_eval<NA, SM, NWARP>(cf, tab, n_terms, S, a);
-                if (!(o.y & 1)) {  // the board stays: remember the outcome, take the step again
-                    known |= 1u << a;
-                    if (o.y & 2)
-                        goal |= 1u << a;
-                    if (lane == a)
-                        rew_lane = o.x;
+            const uint32_t bit = 1u << a;
+            uint32_t *fl = flip_c + (size_t)a * cnw;  // flip planes of the current board and action a
+            int r, goal_left;
+            bool moves;  // the step's own outcome changes the board
+            if (kq & bit) {  // a remembered step that ends in an auto-reset
+                r = __shfl_sync(0xffffffffu, rw, a);
+                goal_left = (gm & bit) != 0u;
+                moves = false;
+            } else if (kc & bit) {  // a remembered step that changes the board
+                r = __shfl_sync(0xffffffffu, rw, a);
+                goal_left = (gm & bit) != 0u;
+                moves = true;
+            } else {
+                const int2 o = memo_step_eval<NA, SM, NWARP>(cf, tab, n_terms, S, a, fl);
+                r = o.x;
+                goal_left = (o.y & 2) != 0;
+                moves = (o.y & 1) != 0;
+                if (lane == a)
+                    rw = r;
+                if (goal_left)
+                    gm |= bit;
+                if (!moves) {  // the board stays: remember the outcome, take the step again
+                    kq |= bit;
                     l0 = e;
                     continue;
                 }
-                r = o.x;
-                t += 1;
-                done = !(o.y & 2) || (cf.max_steps > 0 && t >= cf.max_steps);
-                if (done && cf.auto_reset) {
-                    changed = memo_restore<NWARP>(cf, S.planes, S.basep);
-                    t = 0;
-                } else {
-                    memo_apply<NWARP>(cf, S.planes, S.setp);
-                    changed = 1;
-                }
-            } else {  // a known step that ends in an auto-reset
-                r = __shfl_sync(0xffffffffu, r_l, e);
-                done = 1;
+                kc |= bit;
+            }
+            t += 1;
+            const int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
+            int changed;
+            if (done && cf.auto_reset) {
                 changed = memo_restore<NWARP>(cf, S.planes, S.basep);
                 t = 0;
+            } else {
+                memo_apply<NWARP>(cf, S.planes, fl);
+                changed = moves;
             }
             if (warp == 0 && lane == e) {
                 sum += r;
@@ -524,8 +666,24 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
                     done_traj[(size_t)(b0 + e) * cf.B + env] = (uint8_t)done;
             }
             if (changed) {
-                known = goal = 0;
-                memo_cells<CellT, NA, NWARP>(cf, S.planes, S.cells, v);
+                // the new board goes to the other slot, which becomes the
+                // current one: if it held the same board, its remembered
+                // outcomes hold; else they are dropped
+                const int same = !memo_switch<NWARP>(cf, S.planes, bpl_o) && valid_other;
+                swap_vals(cells_c, cells_o);
+                swap_vals(bpl_c, bpl_o);
+                swap_vals(flip_c, flip_o);
+                swap_vals(kq, okq);
+                swap_vals(kc, okc);
+                swap_vals(gm, ogm);
+                swap_vals(rw, orw);
+                if (same) {
+                    memo_load_cells<NA>(cells_c, n16, v);
+                } else {
+                    kq = kc = gm = 0u;
+                    memo_cells<CellT, NA, NWARP>(cf, S.planes, cells_c, v);
+                }
+                valid_other = 1;
             }
             if (obs_traj && warp == (e % NWARP))
                 memo_store<NA>(obs_env + (size_t)(b0 + e) * step_stride, v, nbytes, obs_mode);
