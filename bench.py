@@ -481,6 +481,7 @@ def time_rollout(args, wl, rank, world, dev, steps, warmup, e2e: bool):
     kernel_ms = sum(ms) / len(ms)
     total_ms = max_over_ranks(sum(ms), world, dev)
     out = dict(rules=rules, cum=cum, fields=fields, seed=seed, env=env, std_path=std_path,
+               path=av.av_rollout_path(env.h),
                kernel_ms=kernel_ms, total_ms=total_ms, wall=wall, clocks=clocks, g0=g0)
     if e2e:
         # the same launch through host buffers (pinned), copies timed
@@ -609,7 +610,7 @@ def run_ours(args, wl):
             "valid_anchor_rule_tests_per_s": value * valid_anchor_rules(wl, m["rules"]),
             "e2e": m["e2e"],
             "roofline": rollout_roofline(av, wl, m, sm_mhz),
-            "gpu_launches": args.steps,
+            "gpu_launches": args.steps * (2 if m["path"] == av.AV_PATH_MEMO else 1),
             "wall_s_timed_region": m["wall"],
         }
         if activity:

@@ -39,6 +39,9 @@ struct av_handle {
     int32_t *d_t = nullptr;
     uint32_t *d_cum = nullptr;
     uint32_t *d_status = nullptr;  // [0] error bits, [1] warning bits
+    uint32_t *d_cost = nullptr;    // [B] memoising rollout: each environment's time in its last launch
+    int32_t *d_order = nullptr;    // [B] memoising rollout: launch order (costliest environments first)
+    bool order_ready = false;      // d_order holds an order (after the first memoising rollout)
     uint64_t *d_vtab = nullptr;     // [B][vis_mask + 1] visited hashes, open addressing (0 = empty)
     uint32_t *d_vzero = nullptr;    // [B] 1 if the state whose hash is 0 was visited
     int32_t *d_n_visited = nullptr; // [B]
@@ -376,6 +379,8 @@ void free_all(av_handle *h)
     cudaFree(h->d_t);
     cudaFree(h->d_cum);
     cudaFree(h->d_status);
+    cudaFree(h->d_cost);
+    cudaFree(h->d_order);
     cudaFree(h->d_vtab);
     cudaFree(h->d_vzero);
     cudaFree(h->d_n_visited);
@@ -533,7 +538,7 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
         (rc = dalloc(h, &h->d_vm, vm.size())) || (rc = dalloc(h, &h->d_masks, masks.size())) ||
         (rc = dalloc(h, (uint8_t **)&h->d_cur, B * h->grid_bytes)) ||
         (rc = dalloc(h, (uint8_t **)&h->d_init, B * h->grid_bytes)) || (rc = dalloc(h, &h->d_t, B)) ||
-        (rc = dalloc(h, &h->d_status, 4)) ||
+        (rc = dalloc(h, &h->d_status, 4)) || (rc = dalloc(h, &h->d_cost, B)) || (rc = dalloc(h, &h->d_order, B)) ||
         (rc = dalloc(h, (uint8_t **)&h->d_rules, (size_t)n_tables * cfg->n_rules * sizeof(av_rule)))) {
         free_all(h);
         delete h;
@@ -687,10 +692,20 @@ int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_tr
                                rew_sum, h->d_status, as_stream(stream));
         return launch_check(h, "variant rollout kernel");
     }
+    // The memoising rollout takes the environments that cost most in its last
+    // launch first (their cost comes mostly from their rules, so it carries
+    // over); the order changes no result, environments being independent.
+    const bool memo = use_memo_rollout(h->cf);
     launch_rollout(h->cf, h->d_arena, h->d_tab_off, h->d_vm, h->d_masks, h->d_cur, h->d_init, h->d_t, n_steps,
                    action_seed, nullptr, obs_traj, rew_traj, done_traj, rew_sum, h->d_status,
-                   as_stream(stream));
-    return launch_check(h, "rollout kernel");
+                   as_stream(stream), memo && h->order_ready ? h->d_order : nullptr, memo ? h->d_cost : nullptr);
+    int rc = launch_check(h, "rollout kernel");
+    if (rc == AV_OK && memo) {
+        launch_memo_order(h->d_cost, h->d_order, h->cf.B, as_stream(stream));
+        rc = launch_check(h, "launch order kernel");
+        h->order_ready = rc == AV_OK;
+    }
+    return rc;
 }
 
 int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_parent,

@@ -46,8 +46,11 @@ struct MemoLayout {
     size_t vm, masks, planes, acc, flip, bplanes, basep, hdr, lead, cells, red, rules, total;
 };
 
-// Warps per environment (CTA): AV_MEMO_WARPS=1|2|4, read by av_create, else 2.
-__host__ __device__ inline int memo_warps(const DevConfig &cf) { return cf.memo_warps == 1 || cf.memo_warps == 4 ? cf.memo_warps : 2; }
+// Warps per environment (CTA): AV_MEMO_WARPS=1|2|4, read by av_create, else 4.
+__host__ __device__ inline int memo_warps(const DevConfig &cf)
+{
+    return cf.memo_warps == 1 || cf.memo_warps == 2 ? cf.memo_warps : 4;
+}
 
 __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool staged)
 {
@@ -491,12 +494,15 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
                     const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
                     const CellT *__restrict__ init, int32_t *tsteps, int n_steps, uint64_t seed,
                     const uint8_t *__restrict__ actions, CellT *obs_traj, int32_t *rew_traj,
-                    uint8_t *done_traj, int32_t *rew_sum, uint32_t *status)
+                    uint8_t *done_traj, int32_t *rew_sum, uint32_t *status, const int32_t *__restrict__ order,
+                    uint32_t *cost)
 {
     constexpr int T = 32 * NWARP;
     extern __shared__ __align__(16) unsigned char smem[];
+    const long long clock0 = clock64();
     const MemoLayout L = memo_layout(cf, SM);
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, env = blockIdx.x;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int env = order ? order[blockIdx.x] : (int)blockIdx.x;
     const int C = cf.C, NW = cf.NW, NWP = cf.NWP, HW = cf.HW, cnw = C * NW;
     const int nbytes = HW * (int)sizeof(CellT);
     MemoSmem S;
@@ -701,9 +707,44 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
                 rew_sum[env] = sum;
             if (warn)
                 atomicOr(status + 1, kWarnAction);
+            if (cost)  // this launch's time for the environment, in units of 256 cycles
+                cost[env] = (uint32_t)min((clock64() - clock0) >> 8, 0xffffffffLL);
         }
     }
 }
+
+#ifdef AV_MEMO_ORDER
+// Launch order of the next memoising rollout (one CTA): environments by
+// decreasing cost in the last launch, in power-of-two buckets (a counting
+// sort; the order within a bucket is arbitrary).  Started first, the costly
+// environments no longer finish after everything else.
+__global__ void __launch_bounds__(1024) memo_order_kernel(const uint32_t *__restrict__ cost, int32_t *order, int B)
+{
+    __shared__ int hist[33], next[33];
+    const int tid = threadIdx.x;
+    if (tid < 33)
+        hist[tid] = 0;
+    __syncthreads();
+    for (int i = tid; i < B; i += blockDim.x)
+        atomicAdd(&hist[32 - __clz(cost[i])], 1);
+    __syncthreads();
+    if (tid == 0) {
+        int s = 0;
+        for (int b = 32; b >= 0; --b) {
+            next[b] = s;
+            s += hist[b];
+        }
+    }
+    __syncthreads();
+    for (int i = tid; i < B; i += blockDim.x)
+        order[atomicAdd(&next[32 - __clz(cost[i])], 1)] = i;
+}
+
+void launch_memo_order(const uint32_t *cost, int32_t *order, int B, cudaStream_t st)
+{
+    memo_order_kernel<<<1, 1024, 0, st>>>(cost, order, B);
+}
+#endif
 
 }  // namespace av
 
@@ -717,23 +758,23 @@ template <typename CellT, int NA, bool SM, int NWARP>
 void memo_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
             const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
             const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
-            uint32_t *status, cudaStream_t st)
+            uint32_t *status, const int32_t *order, uint32_t *cost, cudaStream_t st)
 {
     const size_t sm = memo_layout(cf, SM).total;
     rollout_memo_kernel<CellT, NA, SM, NWARP><<<cf.B, 32 * NWARP, sm, st>>>(
         cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
-        (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
+        (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status, order, cost);
 }
 
 template <typename CellT, int NA, bool SM>
 void memo_w(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
             const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
             const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
-            uint32_t *status, cudaStream_t st)
+            uint32_t *status, const int32_t *order, uint32_t *cost, cudaStream_t st)
 {
 #define AV_MEMO(NWARP)                                                                                     \
     memo_t<CellT, NA, SM, NWARP>(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj, \
-                                 rew_traj, done_traj, rew_sum, status, st)
+                                 rew_traj, done_traj, rew_sum, status, order, cost, st)
     switch (memo_warps(cf)) {
     case 1: AV_MEMO(1); break;
     case 2: AV_MEMO(2); break;
@@ -766,11 +807,12 @@ cudaError_t AV_MEMO_CONFIGURE()
 void AV_MEMO_LAUNCH(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
                     const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
                     const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj,
-                    int32_t *rew_sum, uint32_t *status, cudaStream_t st)
+                    int32_t *rew_sum, uint32_t *status, const int32_t *order, uint32_t *cost, cudaStream_t st)
 {
 #define AV_MEMO(NA, SM)                                                                                  \
     AV_MEMO_NS::memo_w<AV_MEMO_CELL, NA, SM>(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed,   \
-                                             actions, obs_traj, rew_traj, done_traj, rew_sum, status, st)
+                                             actions, obs_traj, rew_traj, done_traj, rew_sum, status, order,  \
+                                             cost, st)
     const bool staged = memo_staged(cf);
     if (cf.NA == 1) {
         if (staged) AV_MEMO(1, true);

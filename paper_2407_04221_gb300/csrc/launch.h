@@ -46,12 +46,15 @@ void launch_rollout_memo_u8(const DevConfig &cf, const uint32_t *arena, const ui
                             const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
                             int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
                             int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
-                            cudaStream_t st);
+                            const int32_t *order, uint32_t *cost, cudaStream_t st);
 void launch_rollout_memo_u16(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
                              const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
                              int32_t *t, int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
                              int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
-                             cudaStream_t st);
+                             const int32_t *order, uint32_t *cost, cudaStream_t st);
+// Next launch order of the memoising rollout from each environment's cost in
+// the last one (k_memo_u16.cu).
+void launch_memo_order(const uint32_t *cost, int32_t *order, int B, cudaStream_t st);
 void launch_rollout_block(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
                           const uint32_t *vm, const uint32_t *masks, void *cur, const void *init, int32_t *t,
                           int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
@@ -136,14 +139,14 @@ inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uin
                            const uint32_t *vm, const uint32_t *masks, void *cur, const void *init, int32_t *t,
                            int n_steps, uint64_t seed, const uint8_t *actions, void *obs_traj,
                            int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
-                           cudaStream_t st)
+                           cudaStream_t st, const int32_t *order = nullptr, uint32_t *cost = nullptr)
 {
     if (use_memo_rollout(cf) && cf.cell_bytes == 1)
         launch_rollout_memo_u8(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
-                               rew_traj, done_traj, rew_sum, status, st);
+                               rew_traj, done_traj, rew_sum, status, order, cost, st);
     else if (use_memo_rollout(cf))
         launch_rollout_memo_u16(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
-                                rew_traj, done_traj, rew_sum, status, st);
+                                rew_traj, done_traj, rew_sum, status, order, cost, st);
     else if (use_env_warp_rollout(cf) && cf.cell_bytes == 1)
         launch_rollout_warp_u8(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
                                rew_traj, done_traj, rew_sum, status, st);
