@@ -35,7 +35,12 @@
  * stream) and returns without synchronising.  Asynchronous CUDA errors are
  * reported by the next call that synchronises (av_sync, av_get_state with a
  * host copy, or any call whose launch fails) as AV_ECUDA; av_last_error()
- * gives the message.  A handle is not thread-safe.
+ * gives the message.  A handle is not thread-safe.  Every call that takes a
+ * handle checks that it is alive (returned by av_create and not yet passed to
+ * av_destroy): a destroyed or never-created pointer gives AV_ESTATE (a NULL
+ * one AV_EINVAL), with no access through it.  av_create returns AV_ENOMEM
+ * when a device allocation fails; setting the environment variable
+ * AV_FAIL_ALLOC makes every such allocation fail, for testing that path.
  *
  * Board layout in memory ("canonical"): [H][W] cell words, row-major, each
  * cell uint8_t when C <= 8, else uint16_t (little-endian), tile bits only.
@@ -55,7 +60,8 @@ enum {
     AV_EINVAL = -1,  /* bad argument, checked before any launch            */
     AV_ENOMEM = -2,  /* device or host allocation failed                   */
     AV_ECUDA = -3,   /* CUDA launch or runtime error                       */
-    AV_ESTATE = -4,  /* call not valid in the handle's state               */
+    AV_ESTATE = -4,  /* call not valid in the handle's state, or the handle
+                        is not alive (destroyed or never created)          */
     AV_EDEVICE = -5  /* a kernel reported an error through its status word */
 };
 
@@ -303,9 +309,12 @@ int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *p
  * Same selection as av_select for boards of batch x H x W cells with C tile
  * channels; the visited sets are caller-owned: visited uint64[batch][capacity]
  * (device, env b's first n_visited[b] entries sorted ascending) and n_visited
- * int32[batch] (device), both updated in place.  status: device uint32 or
- * NULL; receives bit 0 when a visited set would exceed capacity (that env's
- * set is then left unchanged).
+ * int32[batch] (device), both updated in place; entries past an env's new
+ * count are left as they were.  status: device uint32 or NULL; it is
+ * overwritten with this call's bits: bit 0 when a visited set would exceed
+ * capacity (that env's set and count are left unchanged), bit 1 when an
+ * n_visited[b] lies outside 0..capacity (that env selects nothing: n_next[b]
+ * = 0, its frontier zeroed, its set and count left unchanged).
  *
  * The working copy of the visited sets lives in one file-scope device array
  * of AV_SELECT_STATIC_MAX_HASHES hashes that every GPU loading the library

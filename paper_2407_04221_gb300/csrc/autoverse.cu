@@ -16,8 +16,10 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <string>
+#include <unordered_set>
 #include <vector>
 
 #include "launch.h"
@@ -58,6 +60,33 @@ struct av_handle {
 };
 
 namespace {
+
+// Handles alive (created and not yet destroyed): every entry point checks its
+// handle here before touching it, so a destroyed or foreign pointer gives
+// AV_ESTATE instead of a use after free.
+std::mutex g_handles_mu;
+std::unordered_set<const av_handle *> g_handles;
+
+bool handle_live(const av_handle *h)
+{
+    std::lock_guard<std::mutex> lock(g_handles_mu);
+    return g_handles.count(h) != 0;
+}
+
+// AV_EINVAL for a null handle, AV_ESTATE for one that is not alive, else AV_OK.
+int check_handle(const av_handle *h)
+{
+    if (!h)
+        return AV_EINVAL;
+    return handle_live(h) ? AV_OK : AV_ESTATE;
+}
+
+#define AV_HANDLE(h)                        \
+    do {                                    \
+        const int hc_ = check_handle(h);    \
+        if (hc_ != AV_OK)                   \
+            return hc_;                     \
+    } while (0)
 
 int fail(av_handle *h, int code, const std::string &msg)
 {
@@ -419,7 +448,12 @@ const char *av_strerror(int s)
     }
 }
 
-const char *av_last_error(av_handle *h) { return h ? h->last_error.c_str() : "null handle"; }
+const char *av_last_error(av_handle *h)
+{
+    if (!h)
+        return "null handle";
+    return handle_live(h) ? h->last_error.c_str() : "not a live handle (destroyed or never created)";
+}
 
 int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
 {
@@ -481,7 +515,7 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
     // shared memory, or reads them through the L1 cache (default: decided by size).
     if (const char *ms = getenv("AV_MEMO_STAGE"))
         cf.memo_stage = atoi(ms) ? 1 : 2;
-    // AV_MEMO_WARPS=1|2|4: warps per environment of the memoising rollout.
+    // AV_MEMO_WARPS=1|2|4|8: warps per environment of the memoising rollout.
     if (const char *mw = getenv("AV_MEMO_WARPS"))
         cf.memo_warps = atoi(mw);
     if (const char *fw = getenv("AV_FAST_WARPS"))
@@ -598,6 +632,10 @@ int av_create(const av_config *cfg, const av_rule *rules, av_handle **out)
         delete h;
         return AV_ECUDA;
     }
+    {
+        std::lock_guard<std::mutex> lock(g_handles_mu);
+        g_handles.insert(h);
+    }
     *out = h;
     return AV_OK;
 }
@@ -606,6 +644,11 @@ int av_destroy(av_handle *h)
 {
     if (!h)
         return AV_EINVAL;
+    {
+        std::lock_guard<std::mutex> lock(g_handles_mu);
+        if (!g_handles.erase(h))
+            return AV_ESTATE;  // destroyed already, or never created
+    }
     cudaDeviceSynchronize();
     free_all(h);
     delete h;
@@ -614,6 +657,7 @@ int av_destroy(av_handle *h)
 
 int av_reset(av_handle *h, uint64_t seed, void *obs, uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h)
         return AV_EINVAL;
     if (!h->has_cum)
@@ -624,6 +668,7 @@ int av_reset(av_handle *h, uint64_t seed, void *obs, uintptr_t stream)
 
 int av_set_state(av_handle *h, const void *grids, const int32_t *t, int set_as_init, uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || !grids)
         return AV_EINVAL;
     cudaStream_t s = as_stream(stream);
@@ -640,6 +685,7 @@ int av_set_state(av_handle *h, const void *grids, const int32_t *t, int set_as_i
 
 int av_get_state(av_handle *h, void *grids, int32_t *t, uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || !grids)
         return AV_EINVAL;
     cudaStream_t s = as_stream(stream);
@@ -653,6 +699,7 @@ int av_get_state(av_handle *h, void *grids, int32_t *t, uintptr_t stream)
 int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, uint8_t *done,
             uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || !actions)
         return AV_EINVAL;
     if (h->large) {
@@ -675,6 +722,7 @@ int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, ui
 int av_rollout(av_handle *h, int32_t n_steps, uint64_t action_seed, void *obs_traj,
                int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || n_steps < 0)
         return AV_EINVAL;
     if (n_steps == 0)
@@ -712,6 +760,7 @@ int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_par
               void *children, int32_t *rewards, uint8_t *done, uint64_t *hashes,
               uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || F < 0 || (F > 0 && (!parents || !children || !rewards || !hashes)))
         return AV_EINVAL;
     if ((size_t)h->cf.B * (size_t)F > 0x7fffffffu)
@@ -730,6 +779,7 @@ int av_expand(av_handle *h, const void *parents, int32_t F, const int32_t *n_par
 int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, int32_t *player_yx,
                uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || !obs)
         return AV_EINVAL;
     if (window < 1 || window > AV_MAX_WINDOW)
@@ -744,6 +794,7 @@ int av_observe(av_handle *h, const void *grids, int32_t window, uint8_t *obs, in
 
 int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || (!bits && h->cf.R > 0))
         return AV_EINVAL;
     const size_t n = (size_t)h->n_tables * h->cf.R;
@@ -755,6 +806,7 @@ int av_rule_obs(av_handle *h, uint8_t *bits, int32_t *reward, uintptr_t stream)
 
 int av_set_variant(av_handle *h, const av_variant *v)
 {
+    AV_HANDLE(h);
     if (!h)
         return AV_EINVAL;
     VariantParams p{};
@@ -804,6 +856,7 @@ int av_mutate(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t n_rules, c
 int av_search_init(av_handle *h, const void *roots, uint64_t *root_hash, uint8_t *root_live,
                    uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h || !roots || !root_hash || !root_live)
         return AV_EINVAL;
     if (h->host_cfg.search_capacity < 1)
@@ -824,6 +877,7 @@ int av_select(av_handle *h, int32_t F, const int32_t *n_parent, const int32_t *p
               int32_t *next_cum, uint64_t *next_hash, uint8_t *next_live, int32_t *n_next,
               uintptr_t stream)
 {
+    AV_HANDLE(h);
     if (!h)
         return AV_EINVAL;
     if (h->host_cfg.search_capacity < 1)
@@ -931,6 +985,7 @@ int av_select_static(int32_t batch, int32_t H, int32_t W, int32_t C, int32_t F,
 
 int av_sync(av_handle *h)
 {
+    AV_HANDLE(h);
     if (!h)
         return AV_EINVAL;
     AV_CUDA(h, cudaDeviceSynchronize());
@@ -947,6 +1002,7 @@ int av_sync(av_handle *h)
 
 int av_rollout_path(av_handle *h, int32_t *path)
 {
+    AV_HANDLE(h);
     if (!h || !path)
         return AV_EINVAL;
     *path = h->large                   ? AV_PATH_BAND
@@ -960,6 +1016,7 @@ int av_rollout_path(av_handle *h, int32_t *path)
 
 int av_warnings(av_handle *h, uint32_t *bits)
 {
+    AV_HANDLE(h);
     if (!h || !bits)
         return AV_EINVAL;
     AV_CUDA(h, cudaDeviceSynchronize());

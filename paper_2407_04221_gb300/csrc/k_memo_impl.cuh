@@ -46,10 +46,10 @@ struct MemoLayout {
     size_t vm, masks, planes, acc, flip, bplanes, basep, hdr, lead, cells, red, rules, total;
 };
 
-// Warps per environment (CTA): AV_MEMO_WARPS=1|2|4, read by av_create, else 4.
+// Warps per environment (CTA): AV_MEMO_WARPS=1|2|4|8, read by av_create, else 4.
 __host__ __device__ inline int memo_warps(const DevConfig &cf)
 {
-    return cf.memo_warps == 1 || cf.memo_warps == 2 ? cf.memo_warps : 4;
+    return cf.memo_warps == 1 || cf.memo_warps == 2 || cf.memo_warps == 8 ? cf.memo_warps : 4;
 }
 
 __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool staged)
@@ -778,6 +778,7 @@ void memo_w(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
     switch (memo_warps(cf)) {
     case 1: AV_MEMO(1); break;
     case 2: AV_MEMO(2); break;
+    case 8: AV_MEMO(8); break;
     default: AV_MEMO(4); break;
     }
 #undef AV_MEMO
@@ -795,7 +796,8 @@ cudaError_t AV_MEMO_CONFIGURE()
 #define AV_SETM(NA, SM) \
     set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 1>); \
     set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 2>); \
-    set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 4>);
+    set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 4>); \
+    set((const void *)rollout_memo_kernel<AV_MEMO_CELL, NA, SM, 8>);
     AV_SETM(1, true)
     AV_SETM(1, false)
     AV_SETM(2, true)

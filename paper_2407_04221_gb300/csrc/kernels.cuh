@@ -51,6 +51,7 @@ constexpr int kMaxCand = 4096;  // av_select: candidates per env
 constexpr int kActChunk = 256;  // actions drawn ahead, per CTA
 constexpr int kMaxSmemRuleWords = 8192;  // stage a rule table in shared memory up to 32 KiB
 constexpr uint32_t kStatusVisitedOverflow = 1u;
+constexpr uint32_t kStatusVisitedCount = 2u;  // a caller-owned visited count outside 0..capacity
 constexpr uint32_t kWarnAction = 1u;
 constexpr uint32_t kTermAbsent = 0x80000000u;  // flag in a term's shift word
 // One warp per environment: present terms of a rule held in registers, and the
@@ -2111,6 +2112,22 @@ select_kernel(DevConfig cf, int cap, int parity, int F, const int32_t *__restric
     uint64_t *vis_out = visited + ((size_t)(parity ^ 1) * cf.B + b) * cap;
     const int nv = n_visited[b];
     const int np = n_parent[b];
+    if (nv < 0 || nv > cap) {
+        // a count the set cannot hold (block-uniform): nothing of the set is
+        // read as hashes; the env selects nothing and keeps its set as given
+        if (tid == 0) {
+            atomicOr(status, kStatusVisitedCount);
+            n_next[b] = 0;
+        }
+        for (int s = tid; s < k; s += blockDim.x) {
+            next_cum[(size_t)b * k + s] = 0;
+            next_hash[(size_t)b * k + s] = 0;
+            next_live[(size_t)b * k + s] = 0;
+        }
+        for (int i = tid; i < cap; i += blockDim.x)
+            vis_out[i] = vis_in[i];
+        return;
+    }
 
     // 1. candidates that exist and are not yet visited; key (hash, cum desc, index)
     for (int i = tid; i < n2; i += blockDim.x) {
@@ -2210,7 +2227,7 @@ select_kernel(DevConfig cf, int cap, int parity, int F, const int32_t *__restric
             atomicOr(status, kStatusVisitedOverflow);
             n_visited[b] = nv;
         }
-        for (int i = tid; i < nv; i += blockDim.x)
+        for (int i = tid; i < cap; i += blockDim.x)  // the set as given, unused tail included
             vis_out[i] = vis_in[i];
         return;
     }
@@ -2218,6 +2235,8 @@ select_kernel(DevConfig cf, int cap, int parity, int F, const int32_t *__restric
         vis_out[i + lower_bound_u64(sel, take, vis_in[i])] = vis_in[i];
     for (int j = tid; j < take; j += blockDim.x)
         vis_out[j + lower_bound_u64(vis_in, nv, sel[j])] = sel[j];
+    for (int i = nv + take + tid; i < cap; i += blockDim.x)  // the unused tail as given
+        vis_out[i] = vis_in[i];
     if (tid == 0)
         n_visited[b] = nv + take;
 }

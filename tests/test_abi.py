@@ -101,3 +101,34 @@ def test_missing_library_fails_loudly(tmp_path, monkeypatch):
     monkeypatch.setattr(av, "LIB_PATH", str(tmp_path / "absent.so"))
     with pytest.raises(RuntimeError, match="missing"):
         av.load()
+
+
+def test_allocation_failure_gives_enomem(lib, monkeypatch):
+    """AV_FAIL_ALLOC makes av_create's device allocations fail: AV_ENOMEM, and
+    no handle (the refusal comes before any device memory is touched)."""
+    import paper_2407_04221_gb300 as av
+    import workload as wk
+    monkeypatch.setenv("AV_FAIL_ALLOC", "1")
+    fields = dict(batch=4, H=16, W=16, C=4, n_rules=2, rules_per_env=0, max_steps=0, auto_reset=0,
+                  ch_player=2, ch_goal=3, ch_empty=0, ch_wall=1, border_wall=1, cum_per_env=0)
+    cfg = av.AvConfig(**{k: v for k, v in fields.items()})
+    rules = np.ascontiguousarray(wk.base_game_rules(4))
+    h = ctypes.c_void_p()
+    rc = lib.av_create(ctypes.byref(cfg), rules.ctypes.data_as(ctypes.c_void_p), ctypes.byref(h))
+    assert rc == av.AV_ENOMEM
+    assert h.value is None
+
+
+def test_calls_on_a_handle_that_is_not_alive(lib):
+    """A pointer that av_create never returned (or that av_destroy already
+    took) is refused with AV_ESTATE, without being dereferenced."""
+    import paper_2407_04221_gb300 as av
+    fake = ctypes.c_void_p(0x1000)
+    assert lib.av_destroy(fake) == av.AV_ESTATE
+    assert lib.av_sync(fake) == av.AV_ESTATE
+    assert lib.av_step(fake, fake, None, None, None, 0) == av.AV_ESTATE
+    assert lib.av_rollout(fake, 1, 0, None, None, None, None, 0) == av.AV_ESTATE
+    assert lib.av_set_variant(fake, None) == av.AV_ESTATE
+    path = ctypes.c_int32()
+    assert lib.av_rollout_path(fake, ctypes.byref(path)) == av.AV_ESTATE
+    assert b"not a live handle" in lib.av_last_error(fake)

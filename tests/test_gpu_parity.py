@@ -304,3 +304,23 @@ def test_launch_lengths_and_continuation(monkeypatch, path):
         np.testing.assert_array_equal(to_np(t), ref["t"])
         g, t0 = ref["grids"], ref["t"]
     env.close()
+
+
+def test_destroyed_handle_is_refused():
+    """After av_destroy every call on the handle returns AV_ESTATE (the handle
+    is not alive any more), a second av_destroy included."""
+    import ctypes
+
+    import paper_2407_04221_gb300 as av
+    wl = wk.WORKLOADS[2].scaled(batch=4)
+    env, cfg, rules, cum = make(wl, 0)
+    env.reset(5)
+    h = env.h
+    lib = av.load()
+    assert lib.av_destroy(h) == av.AV_OK
+    env.h = None
+    acts = to_dev(np.zeros(4, np.uint8))
+    assert lib.av_step(h, ctypes.c_void_p(acts.data_ptr()), None, None, None, 0) == av.AV_ESTATE
+    assert lib.av_rollout(h, 3, 1, None, None, None, None, 0) == av.AV_ESTATE
+    assert lib.av_sync(h) == av.AV_ESTATE
+    assert lib.av_destroy(h) == av.AV_ESTATE
