@@ -215,19 +215,19 @@ def profile_path(kernel: str, wl) -> str:
     return os.path.join(PROFILE_DIR, f"{kernel}_{wl.name}.md")
 
 
-def profile_traffic(kernel: str, wl, src: str = KERNEL_SRC) -> float | None:
+def source_digest(src) -> str:
+    """sha256 of a kernel's source: one file, or several read in order."""
+    h = hashlib.sha256()
+    for path in ((src,) if isinstance(src, str) else src):
+        h.update(open(path, "rb").read())
+    return h.hexdigest()
+
+
+def profile_traffic(kernel: str, wl, src=KERNEL_SRC) -> float | None:
     """DRAM bytes per launch from the committed ncu summary of this kernel on
-    this workload, if it was taken on the current kernel source `src`."""
-    try:
-        text = open(profile_path(kernel, wl)).read()
-    except OSError:
-        return None
-    m = re.search(r"kernel_source_sha256:\s*([0-9a-f]{16,64})", text)
-    t = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
-    if not m or not t:
-        return None
-    cur = hashlib.sha256(open(src, "rb").read()).hexdigest()
-    return float(t.group(1)) if cur.startswith(m.group(1)) else None
+    this workload, if it was taken on the current kernel source `src` (a path,
+    or a tuple of paths hashed together)."""
+    return profile_field(kernel, wl, "dram_bytes_per_launch", src)
 
 
 def cpu_baseline(wl, rules, cum, cfg, seed, budget_s: float = 12.0, variant=None) -> dict:
@@ -360,7 +360,7 @@ def traj_bytes_per_env_step(wl: wk.Workload) -> int:
     return wl.H * wl.W * wl.cell_bytes + 4 + 1
 
 
-def profile_field(kernel: str, wl, field: str, src: str = KERNEL_SRC) -> float | None:
+def profile_field(kernel: str, wl, field: str, src=KERNEL_SRC) -> float | None:
     """A machine-readable figure of the committed ncu summary of this kernel on
     this workload, if the summary was taken on the current kernel source."""
     try:
@@ -371,14 +371,14 @@ def profile_field(kernel: str, wl, field: str, src: str = KERNEL_SRC) -> float |
     t = re.search(field + r":\s*([0-9.eE+]+)", text)
     if not m or not t:
         return None
-    cur = hashlib.sha256(open(src, "rb").read()).hexdigest()
-    return float(t.group(1)) if cur.startswith(m.group(1)) else None
+    return float(t.group(1)) if source_digest(src).startswith(m.group(1)) else None
 
 
-def kernel_source(path: int, av) -> str:
-    """The source file of the rollout kernel for an av_rollout_path value."""
+def kernel_source(path: int, av):
+    """The source of the rollout kernel for an av_rollout_path value: its file,
+    or its files hashed together."""
     if path == av.AV_PATH_MEMO:
-        return MEMO_SRC
+        return (MEMO_SRC, KERNEL_SRC)
     if path == av.AV_PATH_VARIANT:
         return VARIANT_SRC
     if path == av.AV_PATH_BAND:
@@ -714,6 +714,8 @@ def run_single_step(args, wl):
     if rank == 0:
         peaks = measured_peaks()
         path = av.av_rollout_path(env.h)
+        if path == av.AV_PATH_MEMO and not os.environ.get("AV_KERNEL_PATH"):
+            path = av.AV_PATH_BLOCK  # av_step's default kernel on small boards
         kernel = KERNEL_NAMES[path]
         src = kernel_source(path, av)
         sw = SingleStepName(wl)

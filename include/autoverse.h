@@ -354,8 +354,9 @@ int av_warnings(av_handle *h, uint32_t *bits);
  * most 16 rules) step every environment every step; they run when the
  * environment variable AV_KERNEL_PATH=block|fast|warp|memo, read by av_create,
  * forces a path for tests and measurements.  Every path gives the same
- * results.  Writes the path to *path; AV_EINVAL for a null argument.  No GPU
- * work. */
+ * results.  The path named is av_rollout's; av_step (one step per launch, no
+ * outcome to repeat) takes the block kernel unless AV_KERNEL_PATH forces one.
+ * Writes the path to *path; AV_EINVAL for a null argument.  No GPU work. */
 enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3, AV_PATH_VARIANT = 4, AV_PATH_BAND = 5,
        AV_PATH_MEMO = 6 };
 int av_rollout_path(av_handle *h, int32_t *path);

@@ -141,6 +141,15 @@ inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uin
                            int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum, uint32_t *status,
                            cudaStream_t st, const int32_t *order = nullptr, uint32_t *cost = nullptr)
 {
+    // A launch of one step given its actions (av_step) has no outcome to
+    // repeat: by default it takes the block kernel, whose setup is the
+    // shortest (measured on the 16,384-env training shape: 0.126 ms against
+    // 0.147-0.184 ms for the memoising kernel).
+    if (n_steps == 1 && actions && cf.path == 0) {
+        launch_rollout_block(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
+                             rew_traj, done_traj, rew_sum, status, st);
+        return;
+    }
     if (use_memo_rollout(cf) && cf.cell_bytes == 1)
         launch_rollout_memo_u8(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
                                rew_traj, done_traj, rew_sum, status, order, cost, st);
