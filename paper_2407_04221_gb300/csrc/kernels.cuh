@@ -124,7 +124,7 @@ __host__ __device__ inline StepSmem step_smem(const DevConfig &cf, int n_cell_bo
     s.vm = align16(s.basep + pw);
     s.masks = align16(s.vm + (size_t)kShapes * cf.NW * 4);
     s.red = align16(s.masks + (size_t)3 * cf.NW * 4);
-    s.acts = align16(s.red + (size_t)(kWarps + 4) * 4);
+    s.acts = align16(s.red + (size_t)(kWarps + 16) * 4);
     s.rules = align16(s.acts + kActChunk);
     s.cells = align16(s.rules + (size_t)cf.rule_words * 4);
     s.total = align16(s.cells + (size_t)n_cell_boards * cf.HW * 2);
@@ -134,7 +134,9 @@ __host__ __device__ inline StepSmem step_smem(const DevConfig &cf, int n_cell_bo
 struct Smem {
     uint2 *planes;
     uint32_t *setp, *clrp, *basep, *vm, *masks, *rules;
-    int *red, *flags;
+    int *red, *flags;  // flags: [0] a match this step, [1] action warning, [3] band step reward,
+                       // [4] rollout_kernel's remembered actions, [5] its coming step's action,
+                       // [8 + a] the remembered rewards
     uint8_t *acts;
     uint16_t *cells;
 };
@@ -172,7 +174,7 @@ static __device__ void stage_common(const DevConfig &cf, const Smem &S, const ui
         S.vm[i] = __ldg(vm_g + i);
     for (int i = tid; i < 3 * cf.NW; i += kThreads)
         S.masks[i] = __ldg(masks_g + i);
-    if (tid < kWarps + 4)
+    if (tid < kWarps + 16)
         S.red[tid] = 0;
 }
 
@@ -506,31 +508,61 @@ rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t 
 
     int t = tsteps[env];
     int sum = 0;
-    if (warp == 0)
+    if (warp == 0) {
         write_force(cf, S, S.acts[0]);
+        if (lane == 0)
+            S.flags[5] = S.acts[0];  // the action of the coming step (the ring slot may be refilled)
+    }
     __syncthreads();
 
+    // While the board stays as it is, the step with action a always has the
+    // same outcome: an action whose step matched nothing that changes the board
+    // is remembered (bit a of S.flags[4], its reward in S.flags[8 + a]) and its
+    // later steps skip the match; any change of the board forgets them all.
     for (int s = 0; s < n_steps; ++s) {
         if (((s + 1) & (kActChunk - 1)) == 0)
             fill_actions(actions, seed, env, s + 1, n_steps, S);
-        match_all<NA, SM>(cf, tab, S);
+        const int a = S.flags[5];
+        const bool known = (S.flags[4] >> a) & 1;  // block-uniform (written before the last barrier)
+        if (!known)
+            match_all<NA, SM>(cf, tab, S);
         __syncthreads();
         if (warp == 0) {
-            // combine: a bit changes where any match asks for it (one index over
-            // every channel's words, so small boards keep all lanes busy)
-            if (S.flags[0]) {
-                // (c, w) of index i = c * NW + w, stepped without a division
-                for (int i = lane, c = lane / NW, w = lane - (lane / NW) * NW; i < C * NW; i += 32) {
-                    const uint32_t d = S.planes[c * NWP + w].x, st = S.setp[i], cl = S.clrp[i];
-                    S.setp[i] = 0u;
-                    S.clrp[i] = 0u;
-                    put_word(S.planes, NWP, c, w, (d & ~cl) | (~d & st));
-                    for (w += 32; w >= NW; w -= NW)
-                        ++c;
+            int rew, changed = 0;
+            if (known) {
+                rew = S.flags[8 + a];
+            } else {
+                rew = lane < kWarps ? S.red[lane] : 0;
+                rew = __reduce_add_sync(0xffffffffu, rew);
+                // combine: a bit changes where any match asks for it (one index over
+                // every channel's words, so small boards keep all lanes busy)
+                if (S.flags[0]) {
+                    // (c, w) of index i = c * NW + w, stepped without a division
+                    for (int i = lane, c = lane / NW, w = lane - (lane / NW) * NW; i < C * NW; i += 32) {
+                        const uint32_t d = S.planes[c * NWP + w].x, st = S.setp[i], cl = S.clrp[i];
+                        const uint32_t nd = (d & ~cl) | (~d & st);
+                        S.setp[i] = 0u;
+                        S.clrp[i] = 0u;
+                        if (nd != d) {
+                            changed = 1;
+                            put_word(S.planes, NWP, c, w, nd);
+                        }
+                        for (w += 32; w >= NW; w -= NW)
+                            ++c;
+                    }
+                    changed = __any_sync(0xffffffffu, changed);
+                    __syncwarp();
+                    if (lane == 0)
+                        S.flags[0] = 0;
                 }
-                __syncwarp();
-                if (lane == 0)
-                    S.flags[0] = 0;
+                if (lane == 0) {  // remember the step: it left the board as it was
+                    if (changed) {
+                        S.flags[4] = 0;
+                    } else {
+                        S.flags[4] |= 1 << a;
+                        S.flags[8 + a] = rew;
+                    }
+                }
             }
             int goal = cf.ch_goal < 0;
             if (cf.ch_goal >= 0)
@@ -546,9 +578,9 @@ rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t 
                         ++c;
                 }
                 t = 0;
+                if (lane == 0)
+                    S.flags[4] = 0;  // the board may have changed
             }
-            int rew = lane < kWarps ? S.red[lane] : 0;
-            rew = __reduce_add_sync(0xffffffffu, rew);
             sum += rew;
             if (lane == 0) {
                 if (rew_traj)
@@ -557,8 +589,12 @@ rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t 
                     done_traj[(size_t)s * cf.B + env] = (uint8_t)done;
             }
             __syncwarp();
-            if (s + 1 < n_steps)
-                write_force(cf, S, S.acts[(s + 1) & (kActChunk - 1)]);
+            if (s + 1 < n_steps) {
+                const int a_next = S.acts[(s + 1) & (kActChunk - 1)];
+                write_force(cf, S, a_next);
+                if (lane == 0)
+                    S.flags[5] = a_next;
+            }
         }
         __syncthreads();
         if (obs_traj) {
