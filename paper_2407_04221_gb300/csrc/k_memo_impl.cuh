@@ -27,6 +27,8 @@
 // in each), so all of them reach each block barrier together.
 #pragma once
 
+#include <algorithm>
+
 #include "launch.h"
 
 namespace av {
@@ -73,11 +75,12 @@ __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool stag
 }
 
 // Whether the whole rule table is copied into shared memory: when the
-// environment's region with it still lets as many environments share an SM
-// as the register budget does (32 warps of 64 registers per thread), else the
-// table is read through the L1 cache, and only for rules that pass their
-// leading terms.  AV_MEMO_STAGE=1 (copy) or 0 (do not), read by av_create,
-// forces the choice for measurements.
+// environment's region with it still lets six environments share an SM (the
+// register budget allows eight); else the table is read through the L1 cache,
+// and only for rules that pass their leading terms.  On the trajectory
+// workload (the largest table 31 KB with its region: seven per SM) staging
+// took the launch from 18.3 to 16.1 ms.  AV_MEMO_STAGE=1 (copy) or 0 (do not),
+// read by av_create, forces the choice for measurements.
 inline bool memo_staged(const DevConfig &cf)
 {
     if (cf.rule_words <= 0 || cf.memo_stage == 2)
@@ -85,7 +88,7 @@ inline bool memo_staged(const DevConfig &cf)
     const size_t total = memo_layout(cf, true).total;
     if (cf.memo_stage == 1)
         return total <= (size_t)kDynSmemLimit;
-    return total * (size_t)(32 / memo_warps(cf)) <= (size_t)224 * 1024;
+    return total * (size_t)std::max(1, 24 / memo_warps(cf)) <= (size_t)227 * 1024;
 }
 
 // This lane's share of a board's canonical bytes to dst (global): 16-byte
