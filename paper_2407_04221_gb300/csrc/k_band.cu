@@ -80,7 +80,7 @@ __global__ void __launch_bounds__(kThreads)
         S.planes[i] = make_uint2(0u, 0u);
     if (SM)
         stage_rules(tab_g, tab_off[table + 1] - tab_off[table], S.rules);
-    if (tid < kWarps + 4)
+    if (tid < kWarps + 16)
         S.red[tid] = 0;
     fill_actions(actions, seed, env, 0, n_steps, S);
     const CellT *src = cur + (size_t)env * HW, *isrc = init + (size_t)env * HW;
@@ -105,16 +105,26 @@ __global__ void __launch_bounds__(kThreads)
     __syncthreads();
     for (int w = tid; w < NW; w += kThreads)
         P[C * NW + w] = force_word(cf, P + (cf.ch_player >= 0 ? cf.ch_player : 0) * NW, masks_g, NW, w, S.acts[0]);
+    if (tid == 0)
+        S.flags[5] = S.acts[0];  // the action of the coming step (the ring slot may be refilled)
     int t = tsteps[env];
     int sum = 0;
+    int goal_left = 1;  // of the board in hand, once a step has been evaluated on it
+    __shared__ int s_chg;
     __syncthreads();
 
+    // While the board stays as it is, the step with action a always has the
+    // same outcome: an action whose step changed nothing is remembered (bit a
+    // of S.flags[4], its reward in S.flags[8 + a]) and its later steps skip the
+    // bands until the board changes or resets.
     const int n_bands = (H + band_rows - 1) / band_rows;
     for (int s = 0; s < n_steps; ++s) {
         if (((s + 1) & (kActChunk - 1)) == 0)
             fill_actions(actions, seed, env, s + 1, n_steps, S);
+        const int act = S.flags[5];
+        const bool known = (S.flags[4] >> act) & 1;  // block-uniform (written before the last barrier)
         int rew = 0;
-        for (int band = 0; band < n_bands; ++band) {
+        for (int band = 0; known ? false : band < n_bands; ++band) {
             const int A0 = band * band_rows * W, A1 = min(H, (band + 1) * band_rows) * W;  // anchor cells
             const int w0 = A0 >> 5;
             for (int i = tid; i < (C + 1) * NWB; i += kThreads) {
@@ -156,37 +166,55 @@ __global__ void __launch_bounds__(kThreads)
                 S.flags[0] = 0;
         }
         // ---- the whole board: combine, goal test, reset, next force plane
-        if (tid == 0)
-            s_any = 0;
-        __syncthreads();
-        int goal = 0;
-        for (int i = tid; i < C * NW; i += kThreads) {
-            uint32_t d = P[i];
-            const uint32_t st = SETg[i], cl = CLRg[i];
-            if (st | cl) {
-                d = (d & ~cl) | (~d & st);
-                P[i] = d;
-                SETg[i] = 0u;
-                CLRg[i] = 0u;
+        if (!known) {
+            if (tid == 0) {
+                s_any = 0;
+                s_chg = 0;
             }
-            if (cf.ch_goal >= 0 && i / NW == cf.ch_goal && d)
-                goal = 1;
+            __syncthreads();
+            int goal = 0, chg = 0;
+            for (int i = tid; i < C * NW; i += kThreads) {
+                uint32_t d = P[i];
+                const uint32_t st = SETg[i], cl = CLRg[i];
+                if (st | cl) {
+                    const uint32_t nd = (d & ~cl) | (~d & st);
+                    chg |= nd != d;
+                    d = nd;
+                    P[i] = d;
+                    SETg[i] = 0u;
+                    CLRg[i] = 0u;
+                }
+                if (cf.ch_goal >= 0 && i / NW == cf.ch_goal && d)
+                    goal = 1;
+            }
+            if (goal)
+                s_any = 1;
+            if (chg)
+                s_chg = 1;
+            rew = __reduce_add_sync(0xffffffffu, rew);  // warp 0 holds every warp's share
+            if (tid == 0)
+                S.flags[3] = rew;
+            __syncthreads();
+            goal_left = cf.ch_goal < 0 || s_any;
+            if (tid == 0) {  // remember the step if it left the board as it was
+                if (s_chg) {
+                    S.flags[4] = 0;
+                } else {
+                    S.flags[4] |= 1 << act;
+                    S.flags[8 + act] = rew;
+                }
+            }
         }
-        if (goal)
-            s_any = 1;
-        rew = __reduce_add_sync(0xffffffffu, rew);  // warp 0 holds every warp's share
-        if (tid == 0)
-            S.flags[3] = rew;
-        __syncthreads();
-        const int goal_left = cf.ch_goal < 0 || s_any;
         t += 1;
         const int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
         if (done && cf.auto_reset) {
             for (int i = tid; i < C * NW; i += kThreads)
                 P[i] = BASE[i];
             t = 0;
+            if (tid == 0)
+                S.flags[4] = 0;  // the board may have changed
         }
-        const int step_rew = S.flags[3];
+        const int step_rew = known ? S.flags[8 + act] : S.flags[3];
         sum += step_rew;
         if (tid == 0) {
             if (rew_traj)
@@ -199,6 +227,8 @@ __global__ void __launch_bounds__(kThreads)
             const int a = S.acts[(s + 1) & (kActChunk - 1)];
             for (int w = tid; w < NW; w += kThreads)
                 P[C * NW + w] = force_word(cf, P + (cf.ch_player >= 0 ? cf.ch_player : 0) * NW, masks_g, NW, w, a);
+            if (tid == 0)
+                S.flags[5] = a;
         }
         if (obs_traj) {
             CellT *o = obs_traj + ((size_t)s * cf.B + env) * HW;

@@ -183,3 +183,35 @@ def test_observation_of_large_boards(H, W, C, window):
     np.testing.assert_array_equal(to_np(obs), want)
     np.testing.assert_array_equal(to_np(pyx), want_pyx)
     env.close()
+
+
+def test_remembered_steps_on_large_boards():
+    """The maze game (move and eat rules) on 72 x 72 boards: a push into a wall
+    leaves the board as it is (the band kernel remembers that action's outcome
+    and skips the bands next time), a move or a meal changes it (everything
+    remembered is dropped).  Trajectories against the oracle, bit-exact."""
+    import paper_2407_04221_gb300 as av
+    H = W = 72
+    C, n, steps = 4, 6, 60
+    rules = wk.base_game_rules(C)[None]
+    fields = dict(batch=n, H=H, W=W, C=C, n_rules=2, rules_per_env=0, max_steps=25, auto_reset=1,
+                  ch_player=2, ch_goal=3, ch_empty=0, ch_wall=1, border_wall=0, cum_per_env=0)
+    rng = np.random.default_rng(72)
+    g = np.where(rng.random((n, H, W)) < 0.3, 2, 1).astype(np.uint8)  # walls and floor
+    g[:, rng.random((H, W)) < 0.02] = 8  # food
+    for e in range(n):
+        y, x = 10 + 7 * e, 20 + 3 * e
+        g[e, y, x] = 1 | 4
+    env = av.Env(fields, rules)
+    assert av.av_rollout_path(env.h) == av.AV_PATH_BAND
+    env.set_state(to_dev(g), set_as_init=True)
+    res = env.rollout(steps, 5, trajectory=True)
+    cfg = oracle.make_cfg(**fields)
+    ref = oracle.rollout(cfg, rules, g, g, np.zeros(n, np.int32), steps, 5, trajectory=True)
+    np.testing.assert_array_equal(to_np(res["obs"]), ref["obs"])
+    np.testing.assert_array_equal(to_np(res["rew"]), ref["rew"])
+    np.testing.assert_array_equal(to_np(res["done"]), ref["done"])
+    obs = ref["obs"]
+    moved = (obs[1:] != obs[:-1]).reshape(steps - 1, n, -1).any(-1)
+    assert 0.1 < moved.mean() < 0.95  # both kinds of step occur
+    env.close()
