@@ -69,7 +69,7 @@ __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool stag
     L.lead = align16(L.hdr + (size_t)cf.R * 32);
     L.cells = align16(L.lead + (size_t)cf.R * 4 * kMemoLead * 8);
     L.red = align16(L.cells + 2 * align16((size_t)cf.HW * cf.cell_bytes));
-    L.rules = align16(L.red + 16 * 4);
+    L.rules = align16(L.red + 64 * 4);
     L.total = align16(L.rules + (staged ? (size_t)cf.rule_words * 4 : 0));
     return L;
 }
@@ -138,8 +138,9 @@ struct MemoSmem {
     uint32_t *flip;     // [slot][action][C * NW]: the bits each remembered step flips
     uint32_t *bplanes;  // [slot][C * NW]: each slot's board
     uint32_t *basep, *vm, *masks, *cells;
-    int *red;           // [w] reward of warp w's rules; [8] a bit flips; [9] a goal tile is left;
-                        // [10], [11] rules 0-31 / 32-63 that pass their leading terms
+    int *red;  // two sets of 32 (alternate evaluations): [w] the reward of warp w's rules,
+               // [8 + w] warp w's flags (bit 0: a bit flips, bit 1: a goal tile is left),
+               // [16], [17] rules 0-31 / 32-63 that pass their leading terms
     const uint4 *hdr;   // [R][2]: (n_present, n_absent, n_out, reward), (first term, first output, shapes, 0)
     const uint2 *lead;  // [R][4 rotations][kMemoLead] term descriptors
 };
@@ -167,6 +168,51 @@ __device__ __forceinline__ void memo_lead(const DevConfig &cf, const MemoSmem &S
             x &= __funnelshift_r(w.x, w.y, dy[j]) ^ (uint32_t)((int32_t)dy[j] >> 31);
         }
         m[u] = x;
+    }
+}
+
+// memo_lead for rules r0, r0 + step, ..., KB of them at once (all their loads
+// issued before any test, so the warp has independent work while it waits);
+// rules past the table's end give no anchors.
+template <int NA, int KB>
+__device__ __forceinline__ void memo_lead_batch(const DevConfig &cf, const MemoSmem &S, uint32_t pbase, int r0,
+                                                int step, uint32_t (&m)[KB][NA])
+{
+    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    uint32_t shapes[KB];
+    uint4 d01[KB], d23[KB];
+    bool ok[KB];
+#pragma unroll
+    for (int k = 0; k < KB; ++k) {
+        ok[k] = r0 + k * step < cf.R;
+        const int r = ok[k] ? r0 + k * step : r0;
+        shapes[k] = S.hdr[2 * r + 1].z;
+        d01[k] = *reinterpret_cast<const uint4 *>(S.lead + (r * 4 + g) * kMemoLead);
+        d23[k] = *reinterpret_cast<const uint4 *>(S.lead + (r * 4 + g) * kMemoLead + 2);
+    }
+#pragma unroll
+    for (int k = 0; k < KB; ++k) {
+        const uint32_t *vmr = S.vm + ((shapes[k] >> (8 * g)) & 0xffu) * cf.NW;
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            const int a = q + 8 * u;
+            m[k][u] = ok[k] && a < cf.NW ? vmr[a] : 0u;
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < KB; ++k) {
+        const uint32_t dx[4] = {d01[k].x, d01[k].z, d23[k].x, d23[k].z};
+        const uint32_t dy[4] = {d01[k].y, d01[k].w, d23[k].y, d23[k].w};
+#pragma unroll
+        for (int u = 0; u < NA; ++u) {
+            uint32_t x = m[k][u];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint2 w = lds2(pbase + dx[j] + 64 * u);
+                x &= __funnelshift_r(w.x, w.y, dy[j]) ^ (uint32_t)((int32_t)dy[j] >> 31);
+            }
+            m[k][u] = x;
+        }
     }
 }
 
@@ -238,33 +284,43 @@ __device__ __forceinline__ void memo_write(const DevConfig &cf, const uint4 *op,
 // inlined: it runs once per board and action.
 template <int NA, bool SM, int NWARP>
 static __device__ __forceinline__ int2 memo_step_eval(DevConfig cf, const uint32_t *tab, uint32_t n_terms, MemoSmem S,
-                                                       int a, uint32_t *flip_out)
+                                                       int a, uint32_t *flip_out, int &parity)
 {
     constexpr int T = 32 * NWARP;
+    constexpr int KB = 3;  // rules per warp whose leading terms are tested together
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 3, q = lane & 7;
     const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
+    // the reductions alternate between two sets, so that no barrier is needed
+    // after their last read: the set written here was last read two
+    // evaluations ago, before the barriers of the one in between
+    int *red = S.red + 32 * parity;
+    parity ^= 1;
     for (int i = tid; i < 2 * NWARP * cnw; i += T)
         S.acc[i] = 0u;
-    if (tid < 16)
-        S.red[tid] = 0;
+    if (tid < 2)
+        red[16 + tid] = 0;
     if (warp == NWARP - 1)
         force_plane(cf, S.planes, S.masks, a);
     __syncthreads();
     const uint32_t pbase = (uint32_t)__cvta_generic_to_shared(S.planes) + q * 8;
     // this warp's rules whose leading terms pass somewhere
     uint32_t alive0 = 0, alive1 = 0;
-#pragma unroll 2
-    for (int r = warp; r < cf.R; r += NWARP) {
-        uint32_t m[NA], any = 0;
-        memo_lead<NA>(cf, S, pbase, r, m);
+    for (int r0 = warp; r0 < cf.R; r0 += KB * NWARP) {
+        uint32_t m[KB][NA];
+        memo_lead_batch<NA, KB>(cf, S, pbase, r0, NWARP, m);
 #pragma unroll
-        for (int u = 0; u < NA; ++u)
-            any |= m[u];
-        if (any) {
-            if (r < 32)
-                alive0 |= 1u << r;
-            else
-                alive1 |= 1u << (r - 32);
+        for (int k = 0; k < KB; ++k) {
+            uint32_t any = 0;
+#pragma unroll
+            for (int u = 0; u < NA; ++u)
+                any |= m[k][u];
+            const int r = r0 + k * NWARP;
+            if (any) {  // (rules past the end have no anchors)
+                if (r < 32)
+                    alive0 |= 1u << r;
+                else
+                    alive1 |= 1u << (r - 32);
+            }
         }
     }
     alive0 = __reduce_or_sync(0xffffffffu, alive0);
@@ -273,12 +329,12 @@ static __device__ __forceinline__ int2 memo_step_eval(DevConfig cf, const uint32
         // the rules that passed, dealt out afresh: the k-th of them to warp k mod NWARP
         if (lane == 0) {
             if (alive0)
-                atomicOr(reinterpret_cast<unsigned int *>(S.red) + 10, alive0);
+                atomicOr(reinterpret_cast<unsigned int *>(red) + 16, alive0);
             if (alive1)
-                atomicOr(reinterpret_cast<unsigned int *>(S.red) + 11, alive1);
+                atomicOr(reinterpret_cast<unsigned int *>(red) + 17, alive1);
         }
         __syncthreads();
-        const uint32_t all0 = (uint32_t)S.red[10], all1 = (uint32_t)S.red[11];
+        const uint32_t all0 = (uint32_t)red[16], all1 = (uint32_t)red[17];
         alive0 = alive1 = 0;
         int k = 0;
         for (uint32_t x = all0; x; x &= x - 1, ++k)
@@ -337,7 +393,7 @@ static __device__ __forceinline__ int2 memo_step_eval(DevConfig cf, const uint32
     }
     rew = __reduce_add_sync(0xffffffffu, rew);
     if (lane == 0)
-        S.red[warp] = rew;
+        red[warp] = rew;
     __syncthreads();  // every warp's SET / CLEAR bits and reward
     uint32_t any = 0, goal = 0;
     for (int i = tid, c = tid / NW, w = tid - (tid / NW) * NW; i < cnw; i += T, c += T / NW, w += T % NW) {
@@ -360,37 +416,41 @@ static __device__ __forceinline__ int2 memo_step_eval(DevConfig cf, const uint32
     }
     any = __any_sync(0xffffffffu, any != 0u);
     goal = __any_sync(0xffffffffu, goal != 0u);
-    if (lane == 0 && any)
-        atomicOr(S.red + 8, 1);
-    if (lane == 0 && goal)
-        atomicOr(S.red + 9, 1);
+    if (lane == 0)
+        red[8 + warp] = (any ? 1 : 0) | (goal ? 2 : 0);
     __syncthreads();  // the flip planes and flags
-    int total = 0;
+    int total = 0, flags = 0;
 #pragma unroll
-    for (int w = 0; w < NWARP; ++w)
-        total += S.red[w];
-    const int bits = (S.red[8] ? 1 : 0) | ((cf.ch_goal < 0 || S.red[9]) ? 2 : 0);
-    __syncthreads();  // every thread has read the reductions before they are reused
+    for (int w = 0; w < NWARP; ++w) {
+        total += red[w];
+        flags |= red[8 + w];
+    }
+    const int bits = (flags & 1) | ((cf.ch_goal < 0 || (flags & 2)) ? 2 : 0);
     return make_int2(total, bits);
 }
 
-// The board after its step: planes ^= flip (all warps).
+// The board after its step (planes ^= flip), written also into `bpl` (the
+// other slot's flat planes), in one pass (all warps); returns whether it
+// differs from what `bpl` held (every thread).
 template <int NWARP>
-static __device__ __forceinline__ void memo_apply(DevConfig cf, uint2 *planes, const uint32_t *flip)
+static __device__ __forceinline__ int memo_apply_switch(const DevConfig &cf, uint2 *planes, const uint32_t *flip,
+                                                         uint32_t *bpl)
 {
-    const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW;
     constexpr int T = 32 * NWARP;
-    const int tid = threadIdx.x;
+    const int NW = cf.NW, NWP = cf.NWP, cnw = cf.C * NW, tid = threadIdx.x;
+    int diff = 0;
     for (int i = tid, c = tid / NW, w = tid - (tid / NW) * NW; i < cnw; i += T, c += T / NW, w += T % NW) {
         if (w >= NW) {
             w -= NW;
             ++c;
         }
-        const uint32_t f = flip[i];
+        const uint32_t f = flip[i], x = planes[c * NWP + w].x ^ f;
         if (f)
-            put_word(planes, NWP, c, w, planes[c * NWP + w].x ^ f);
+            put_word(planes, NWP, c, w, x);
+        diff |= bpl[i] != x;
+        bpl[i] = x;
     }
-    __syncthreads();
+    return __syncthreads_or(diff);
 }
 
 // Auto-reset: the initial map's planes back into the tile planes (all warps).
@@ -586,6 +646,7 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
     uint32_t *flip_c = S.flip, *flip_o = S.flip + 5 * cnw;
     uint32_t kq = 0u, kc = 0u, gm = 0u, okq = 0u, okc = 0u, ogm = 0u;
     int rw = 0, orw = 0, valid_other = 0;
+    int parity = 0;  // which set of reduction slots the next evaluation uses
     memo_switch<NWARP>(cf, S.planes, bpl_c);
     memo_cells<CellT, NA, NWARP>(cf, S.planes, cells_c, v);
     int t = tsteps[env];
@@ -642,7 +703,7 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
                 goal_left = (gm & bit) != 0u;
                 moves = true;
             } else {
-                const int2 o = memo_step_eval<NA, SM, NWARP>(cf, tab, n_terms, S, a, fl);
+                const int2 o = memo_step_eval<NA, SM, NWARP>(cf, tab, n_terms, S, a, fl, parity);
                 r = o.x;
                 goal_left = (o.y & 2) != 0;
                 moves = (o.y & 1) != 0;
@@ -659,13 +720,13 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
             }
             t += 1;
             const int done = !goal_left || (cf.max_steps > 0 && t >= cf.max_steps);
-            int changed;
+            int changed, diff_other = -1;  // whether the new board differs from the other slot's
             if (done && cf.auto_reset) {
                 changed = memo_restore<NWARP>(cf, S.planes, S.basep);
                 t = 0;
-            } else {
-                memo_apply<NWARP>(cf, S.planes, fl);
-                changed = moves;
+            } else {  // (a board-changing outcome: `moves` holds)
+                diff_other = memo_apply_switch<NWARP>(cf, S.planes, fl, bpl_o);
+                changed = 1;
             }
             if (warp == 0 && lane == e) {
                 sum += r;
@@ -678,7 +739,8 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
                 // the new board goes to the other slot, which becomes the
                 // current one: if it held the same board, its remembered
                 // outcomes hold; else they are dropped
-                const int same = !memo_switch<NWARP>(cf, S.planes, bpl_o) && valid_other;
+                const int same =
+                    !(diff_other >= 0 ? diff_other : memo_switch<NWARP>(cf, S.planes, bpl_o)) && valid_other;
                 swap_vals(cells_c, cells_o);
                 swap_vals(bpl_c, bpl_o);
                 swap_vals(flip_c, flip_o);
