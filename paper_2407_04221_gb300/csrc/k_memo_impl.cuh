@@ -45,7 +45,7 @@ constexpr int kMemoLead = 4;  // leading terms of each rule tested for all rules
 // two header words (uint4 each) and its first kMemoLead terms in each rotation;
 // per-warp reductions; the whole rule table when staged.
 struct MemoLayout {
-    size_t vm, masks, planes, acc, flip, bplanes, basep, hdr, lead, cells, red, rules, total;
+    size_t vm, masks, planes, acc, flip, bplanes, basep, hdr, lead, leadm, cells, red, rules, total;
 };
 
 // Warps per environment (CTA): AV_MEMO_WARPS=1|2|4|8, read by av_create, else 4.
@@ -67,7 +67,8 @@ __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool stag
     L.basep = align16(L.bplanes + 2 * pw);
     L.hdr = align16(L.basep + pw);
     L.lead = align16(L.hdr + (size_t)cf.R * 32);
-    L.cells = align16(L.lead + (size_t)cf.R * 4 * kMemoLead * 8);
+    L.leadm = align16(L.lead + (size_t)cf.R * 4 * kMemoLead * 8);
+    L.cells = align16(L.leadm + (size_t)cf.R * 32 * cf.NA * 4);
     L.red = align16(L.cells + 2 * align16((size_t)cf.HW * cf.cell_bytes));
     L.rules = align16(L.red + 64 * 4);
     L.total = align16(L.rules + (staged ? (size_t)cf.rule_words * 4 : 0));
@@ -143,37 +144,14 @@ struct MemoSmem {
                // [16], [17] rules 0-31 / 32-63 that pass their leading terms
     const uint4 *hdr;   // [R][2]: (n_present, n_absent, n_out, reward), (first term, first output, shapes, 0)
     const uint2 *lead;  // [R][4 rotations][kMemoLead] term descriptors
+    uint32_t *leadm;    // [R][32 lanes][NA]: the anchors that pass each rule's leading terms
 };
 
-// Anchors of this lane's words at which rule r's first kMemoLead terms pass
-// (the valid-anchor mask of the lane's rotation ANDed with each term's
-// shifted plane word, absent terms complemented).
-template <int NA>
-__device__ __forceinline__ void memo_lead(const DevConfig &cf, const MemoSmem &S, uint32_t pbase, int r,
-                                          uint32_t (&m)[NA])
-{
-    const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
-    const uint32_t shapes = S.hdr[2 * r + 1].z;
-    const uint32_t *vmr = S.vm + ((shapes >> (8 * g)) & 0xffu) * cf.NW;
-    const uint4 d01 = *reinterpret_cast<const uint4 *>(S.lead + (r * 4 + g) * kMemoLead);
-    const uint4 d23 = *reinterpret_cast<const uint4 *>(S.lead + (r * 4 + g) * kMemoLead + 2);
-    const uint32_t dx[4] = {d01.x, d01.z, d23.x, d23.z}, dy[4] = {d01.y, d01.w, d23.y, d23.w};
-#pragma unroll
-    for (int u = 0; u < NA; ++u) {
-        const int a = q + 8 * u;
-        uint32_t x = a < cf.NW ? vmr[a] : 0u;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const uint2 w = lds2(pbase + dx[j] + 64 * u);
-            x &= __funnelshift_r(w.x, w.y, dy[j]) ^ (uint32_t)((int32_t)dy[j] >> 31);
-        }
-        m[u] = x;
-    }
-}
-
-// memo_lead for rules r0, r0 + step, ..., KB of them at once (all their loads
-// issued before any test, so the warp has independent work while it waits);
-// rules past the table's end give no anchors.
+// Anchors of this lane's words at which the first kMemoLead terms of rules r0,
+// r0 + step, ... (KB of them) pass: the valid-anchor mask of the lane's
+// rotation ANDed with each term's shifted plane word, absent terms
+// complemented.  All loads are issued before any test, so the warp has
+// independent work while it waits; rules past the table's end give no anchors.
 template <int NA, int KB>
 __device__ __forceinline__ void memo_lead_batch(const DevConfig &cf, const MemoSmem &S, uint32_t pbase, int r0,
                                                 int step, uint32_t (&m)[KB][NA])
@@ -315,6 +293,11 @@ static __device__ __forceinline__ int2 memo_step_eval(DevConfig cf, const uint32
             for (int u = 0; u < NA; ++u)
                 any |= m[k][u];
             const int r = r0 + k * NWARP;
+            if (r < cf.R) {
+#pragma unroll
+                for (int u = 0; u < NA; ++u)  // kept for the warp that takes the rule on
+                    S.leadm[(r * 32 + lane) * NA + u] = m[k][u];
+            }
             if (any) {  // (rules past the end have no anchors)
                 if (r < 32)
                     alive0 |= 1u << r;
@@ -354,7 +337,9 @@ static __device__ __forceinline__ int2 memo_step_eval(DevConfig cf, const uint32
             const int r = 32 * k + __ffs(alive) - 1;
             alive &= alive - 1;
             uint32_t m[NA];
-            memo_lead<NA>(cf, S, pbase, r, m);
+#pragma unroll
+            for (int u = 0; u < NA; ++u)  // written by the warp that tested the leading terms
+                m[u] = S.leadm[(r * 32 + lane) * NA + u];
             const uint4 h0 = S.hdr[2 * r], h1 = S.hdr[2 * r + 1];
             const uint32_t nt = h0.x + h0.y;
             const uint2 *tp = terms + (size_t)h1.x * 4 + g;
@@ -582,6 +567,7 @@ rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint
     uint2 *lead = reinterpret_cast<uint2 *>(smem + L.lead);
     S.hdr = hdr;
     S.lead = lead;
+    S.leadm = reinterpret_cast<uint32_t *>(smem + L.leadm);
     const int table = cf.rules_per_env ? env : 0;
     const uint32_t *tab_g = arena + tab_off[table];
     const uint32_t *tab = SM ? reinterpret_cast<const uint32_t *>(smem + L.rules) : tab_g;
