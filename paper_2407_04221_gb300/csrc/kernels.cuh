@@ -2089,24 +2089,70 @@ __device__ __forceinline__ bool key_less(const Key128 &a, const Key128 &b)
     return a.hi < b.hi || (a.hi == b.hi && a.lo < b.lo);
 }
 
-// Block-wide bitonic sort of n2 (power of two) keys in shared memory, ascending.
+// One compare-exchange of a bitonic stage (block k, partner distance j): keys
+// i and i ^ j, ascending where bit k of i is clear.
+__device__ __forceinline__ void bitonic_cmpx(Key128 *keys, int i, int k, int j)
+{
+    const int ixj = i | j;
+    const bool up = (i & k) == 0;
+    const Key128 x = keys[i], y = keys[ixj];
+    if (key_less(y, x) == up) {
+        keys[i] = y;
+        keys[ixj] = x;
+    }
+}
+
+// Lower key of the p-th compare-exchange pair of stage distance j within the
+// 64-key chunk c.
+__device__ __forceinline__ int bitonic_pair(int c, int p, int j)
+{
+    return (c << 6) | ((p & ~(j - 1)) << 1) | (p & (j - 1));
+}
+
+// Block-wide bitonic sort of n2 (power of two) keys in shared memory,
+// ascending; returns after a block barrier.  Stages whose partners lie within
+// one 64-key chunk (distance 32 or less) run warp by warp: warp w owns the
+// chunks w, w + warps, ... and syncs only itself, so of the log2(n2) (log2(n2)
+// + 1) / 2 stages only those of distance 64 or more wait for the whole block
+// (15 of 66 for 2048 keys).  blockDim.x is a multiple of 32.
 static __device__ void bitonic_sort(Key128 *keys, int n2)
 {
-    for (int k = 2; k <= n2; k <<= 1)
-        for (int j = k >> 1; j > 0; j >>= 1) {
-            for (int i = threadIdx.x; i < n2; i += blockDim.x) {
-                const int ixj = i ^ j;
-                if (ixj > i) {
-                    const bool up = (i & k) == 0;
-                    Key128 x = keys[i], y = keys[ixj];
-                    if (key_less(y, x) == up) {
-                        keys[i] = y;
-                        keys[ixj] = x;
-                    }
-                }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+    const int nch = n2 >> 6;  // 64-key chunks
+    if (nch == 0) {  // fewer than 64 keys: every stage block-wide
+        for (int k = 2; k <= n2; k <<= 1)
+            for (int j = k >> 1; j > 0; j >>= 1) {
+                for (int i = threadIdx.x; i < n2; i += blockDim.x)
+                    if ((i & j) == 0)
+                        bitonic_cmpx(keys, i, k, j);
+                __syncthreads();
             }
+        __syncthreads();
+        return;
+    }
+    // blocks of up to 64 keys: each chunk sorted by its warp, alternately
+    // ascending and descending (the direction bit k of the key index)
+    for (int c = warp; c < nch; c += nwarp)
+        for (int k = 2; k <= 64; k <<= 1)
+            for (int j = k >> 1; j > 0; j >>= 1) {
+                bitonic_cmpx(keys, bitonic_pair(c, lane, j), k, j);
+                __syncwarp();
+            }
+    __syncthreads();
+    for (int k = 128; k <= n2; k <<= 1) {
+        for (int j = k >> 1; j >= 64; j >>= 1) {
+            for (int i = threadIdx.x; i < n2; i += blockDim.x)
+                if ((i & j) == 0)
+                    bitonic_cmpx(keys, i, k, j);
             __syncthreads();
         }
+        for (int c = warp; c < nch; c += nwarp)
+            for (int j = 32; j > 0; j >>= 1) {
+                bitonic_cmpx(keys, bitonic_pair(c, lane, j), k, j);
+                __syncwarp();
+            }
+        __syncthreads();
+    }
 }
 
 __device__ __forceinline__ uint32_t cum_desc_key(int32_t cum)
@@ -2431,24 +2477,32 @@ select_hash_kernel(DevConfig cf, int cap, uint32_t vmask, int F, const int32_t *
     }
     __syncthreads();
 
-    // 2. distinct candidates keyed (cum desc, hash, index); one sort
-    for (uint32_t i = tid; i <= T; i += blockDim.x) {
-        uint64_t hsh;
-        unsigned long long v;
+    // 2. distinct candidates keyed (cum desc, hash, index), packed by warps
+    //    (their order before the sort does not matter: the keys are distinct)
+    const int lane = tid & 31;
+    for (uint32_t i0 = tid & ~31u; i0 <= T; i0 += blockDim.x) {
+        const uint32_t i = i0 + lane;
+        uint64_t hsh = 0ull;
+        unsigned long long v = ~0ull;
+        bool have = false;
         if (i < T) {
             hsh = skey[i];
             v = sval[i];
-            if (hsh == 0ull)
-                continue;
-        } else {
+            have = hsh != 0ull;
+        } else if (i == T) {
             v = s_zero_val;
-            hsh = 0ull;
-            if (v == ~0ull)
-                continue;
+            have = v != ~0ull;
         }
-        const int pos = atomicAdd(&s_count, 1);
-        keys[pos].hi = ((v >> 32) << 32) | (hsh >> 32);
-        keys[pos].lo = (hsh << 32) | (v & 0xffffffffull);
+        const uint32_t m = __ballot_sync(0xffffffffu, have);
+        int base = 0;
+        if (lane == 0 && m)
+            base = atomicAdd(&s_count, __popc(m));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (have) {
+            const int pos = base + __popc(m & ((1u << lane) - 1u));
+            keys[pos].hi = ((v >> 32) << 32) | (hsh >> 32);
+            keys[pos].lo = (hsh << 32) | (v & 0xffffffffull);
+        }
     }
     __syncthreads();
     const int nu = s_count;
