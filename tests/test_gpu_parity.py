@@ -86,6 +86,36 @@ def test_rollout_small_full_compare(key, batch, steps):
     env.close()
 
 
+@pytest.mark.parametrize("key,n_sample,steps", [(2, 64, 200), (5, 6, 40), (6, 2, 10)])
+def test_full_size_with_firing_rules(key, n_sample, steps):
+    """The full batch and board of the 1024-env, 64 x 64 and 256 x 256
+    workloads, with rule entries sparse enough (3 % present, 2 % absent per
+    window cell and channel) that rules match and boards change on most steps:
+    the workloads' own random rules almost never match, so this is the
+    full-size check of the match and apply path on those launch shapes (the
+    memoising, block and band kernels)."""
+    wl = wk.WORKLOADS[key].scaled(p_present=0.03, p_absent=0.02)
+    env, cfg, rules, cum = make(wl, 7)
+    s = wk.seeds(7)
+    g0 = to_np(env.reset(s["reset"]))
+    ids = sample_envs(wl.batch, n_sample, seed=key + 10)
+    res = env.rollout(steps, s["actions"], trajectory=True)
+    ref = _oracle_rollout(cfg, rules, g0, ids, steps, s["actions"], trajectory=True)
+    idt = torch.from_numpy(ids).cuda()
+    np.testing.assert_array_equal(to_np(res["obs"].index_select(1, idt)), ref["obs"])
+    np.testing.assert_array_equal(to_np(res["rew"].index_select(1, idt)), ref["rew"])
+    np.testing.assert_array_equal(to_np(res["done"].index_select(1, idt)), ref["done"])
+    np.testing.assert_array_equal(to_np(res["rew_sum"])[ids], ref["rew_sum"])
+    g, t = env.get_state()
+    np.testing.assert_array_equal(to_np(g)[ids], ref["grids"])
+    np.testing.assert_array_equal(to_np(t)[ids], ref["t"])
+    prev = np.concatenate([g0[ids][None], ref["obs"][:-1]], 0)
+    assert (ref["obs"] != prev).reshape(steps, len(ids), -1).any(-1).mean() > 0.5  # boards change
+    assert (ref["rew"] != 0).mean() > 0.5  # and matches pay
+    env.sync()
+    env.close()
+
+
 @pytest.mark.parametrize("key,n_sample", [(2, 96), (3, 24), (5, 6)])
 def test_rollout_full_size_sampled(key, n_sample):
     """The benchmark's launch configuration: full batch, full fused length."""
