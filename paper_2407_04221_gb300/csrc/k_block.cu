@@ -7,6 +7,26 @@ namespace {
 
 #define AV_FOR_NA(MACRO, CELL) MACRO(CELL, 1) MACRO(CELL, 2) MACRO(CELL, 4) MACRO(CELL, 8) MACRO(CELL, 16)
 
+template <typename CellT, int NA, bool SM>
+void block_launch(const DevConfig &cf, size_t sm, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+                  const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
+                  const uint8_t *actions, void *obs_traj, int32_t *rew_traj, uint8_t *done_traj, int32_t *rew_sum,
+                  uint32_t *status, cudaStream_t st)
+{
+    // one-step launches of small boards (av_step) take the kernel without runs
+    if constexpr (NA <= 2) {
+        if (n_steps == 1) {
+            rollout_kernel<CellT, NA, SM, false><<<cf.B, kThreads, sm, st>>>(
+                cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
+                (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
+            return;
+        }
+    }
+    rollout_kernel<CellT, NA, SM, true><<<cf.B, kThreads, sm, st>>>(
+        cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
+        (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
+}
+
 template <typename CellT, int NA>
 void block_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
              const uint32_t *masks, void *cur, const void *init, int32_t *t, int n_steps, uint64_t seed,
@@ -15,13 +35,11 @@ void block_t(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off
 {
     const size_t sm = step_smem(cf, 0).total;
     if (cf.rule_words > 0)
-        rollout_kernel<CellT, NA, true><<<cf.B, kThreads, sm, st>>>(
-            cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
-            (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
+        block_launch<CellT, NA, true>(cf, sm, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions,
+                                      obs_traj, rew_traj, done_traj, rew_sum, status, st);
     else
-        rollout_kernel<CellT, NA, false><<<cf.B, kThreads, sm, st>>>(
-            cf, arena, tab_off, vm, masks, (CellT *)cur, (const CellT *)init, t, n_steps, seed, actions,
-            (CellT *)obs_traj, rew_traj, done_traj, rew_sum, status);
+        block_launch<CellT, NA, false>(cf, sm, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions,
+                                       obs_traj, rew_traj, done_traj, rew_sum, status, st);
 }
 
 }  // namespace
@@ -34,8 +52,12 @@ cudaError_t configure_block()
             e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmemLimit);
     };
 #define AV_SET(CELL, NA)                                       \
-    set((const void *)rollout_kernel<CELL, NA, true>);         \
-    set((const void *)rollout_kernel<CELL, NA, false>);
+    set((const void *)rollout_kernel<CELL, NA, true, true>);   \
+    set((const void *)rollout_kernel<CELL, NA, false, true>);  \
+    if (NA <= 2) {                                             \
+        set((const void *)rollout_kernel<CELL, NA, true, NA <= 2 ? false : true>);  \
+        set((const void *)rollout_kernel<CELL, NA, false, NA <= 2 ? false : true>); \
+    }
     AV_FOR_NA(AV_SET, uint8_t)
     AV_FOR_NA(AV_SET, uint16_t)
 #undef AV_SET

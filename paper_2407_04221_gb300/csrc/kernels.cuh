@@ -136,7 +136,7 @@ struct Smem {
     uint32_t *setp, *clrp, *basep, *vm, *masks, *rules;
     int *red, *flags;  // flags: [0] a match this step, [1] action warning, [3] band step reward,
                        // [4] rollout_kernel's remembered actions, [5] its coming step's action,
-                       // [8 + a] the remembered rewards
+                       // [6] its run of repeated steps, [8 + a] the remembered rewards
     uint8_t *acts;
     uint16_t *cells;
 };
@@ -282,6 +282,39 @@ __device__ __forceinline__ void store_cells(const DevConfig &cf, const uint2 *db
         } else {
             for (int k = 0; k < kPer && p0 + k < HW; ++k)
                 dst[p0 + k] = (CellT)(v >> (8 * (int)sizeof(CellT) * k));
+        }
+    }
+}
+
+// The board's cells (from the doubled planes) into n consecutive steps of a
+// trajectory: dst0, dst0 + stride, ... (stride in cells; each cell word built
+// once).
+template <typename CellT>
+__device__ __forceinline__ void store_cells_steps(const DevConfig &cf, const uint2 *dbl, CellT *dst0, size_t stride,
+                                                  int n, int tid, int nthreads)
+{
+    constexpr int kPer = 4 / (int)sizeof(CellT);
+    const int HW = cf.HW, NWP = cf.NWP;
+    const int n_words = (HW + kPer - 1) / kPer;
+    const bool aligned = (HW % kPer) == 0 && (reinterpret_cast<uintptr_t>(dst0) & 3u) == 0 &&
+                         (stride * sizeof(CellT)) % 4 == 0;
+    for (int g = tid; g < n_words; g += nthreads) {
+        const int p0 = g * kPer, j = p0 >> 5, b = p0 & 31;
+        uint32_t v = 0;
+        for (int c = 0; c < cf.C; ++c) {
+            const uint32_t x = dbl[c * NWP + j].x >> b;
+            const uint32_t spread = sizeof(CellT) == 1 ? ((x & 0xfu) * 0x00204081u) & 0x01010101u
+                                                       : ((x & 0x3u) * 0x00008001u) & 0x00010001u;
+            v |= spread << c;
+        }
+        for (int k = 0; k < n; ++k) {
+            CellT *dst = dst0 + (size_t)k * stride;
+            if (aligned) {
+                reinterpret_cast<uint32_t *>(dst)[g] = v;
+            } else {
+                for (int i = 0; i < kPer && p0 + i < HW; ++i)
+                    dst[p0 + i] = (CellT)(v >> (8 * (int)sizeof(CellT) * i));
+            }
         }
     }
 }
@@ -480,9 +513,13 @@ __device__ __forceinline__ void fill_actions(const uint8_t *__restrict__ actions
 // ---------------------------------------------------------------- kernels
 // Fused rollout (n_steps >= 1).  With `actions` non-null the action of step
 // s is actions[env] (used by av_step, n_steps = 1); else it is drawn.
-// SM: the env's rule table is staged in shared memory.
-template <typename CellT, int NA, bool SM>
-__global__ void __launch_bounds__(kThreads)
+// SM: the env's rule table is staged in shared memory.  RUNS: runs of
+// repeated steps are walked 32 at a time; the kernel of one-step launches
+// leaves them out and keeps the compiler's own register choice (32 a thread
+// for small boards), the others are held to 32 (small boards, eight CTAs per
+// SM) or 64 registers.
+template <typename CellT, int NA, bool SM, bool RUNS>
+__global__ void __launch_bounds__(kThreads, RUNS ? (NA <= 2 ? 8 : 4) : 0)
 rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
                const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
                const CellT *__restrict__ init, int32_t *tsteps, int n_steps, uint64_t seed,
@@ -520,8 +557,66 @@ rollout_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t 
     // is remembered (bit a of S.flags[4], its reward in S.flags[8 + a]) and its
     // later steps skip the match; any change of the board forgets them all.
     for (int s = 0; s < n_steps; ++s) {
-        if (((s + 1) & (kActChunk - 1)) == 0)
+        const bool refill = ((s + 1) & (kActChunk - 1)) == 0;
+        if (refill)
             fill_actions(actions, seed, env, s + 1, n_steps, S);
+        // A run of repeated steps: from this step on, the steps whose actions
+        // are remembered and that end no episode with an auto-reset take their
+        // remembered rewards without a match or a board update, up to 32 at a
+        // time (lane l of warp 0 takes step s + l) and never up to the last
+        // step of the action ring's chunk (that step refills the ring).  Two
+        // block barriers per run instead of two per step: the first publishes
+        // the run's length once every warp has read this step's action; after
+        // it warp 0 writes the next step's action and force plane, which the
+        // second makes visible.
+        if (RUNS && ((S.flags[4] >> S.flags[5]) & 1)) {  // block-uniform
+            if (refill)
+                __syncthreads();  // the ring's next chunk
+            int a_next = 0;
+            if (warp == 0) {
+                const int lim = min(min(32, n_steps - s), ((s + 1) | (kActChunk - 1)) - s);
+                const int a_l = lane == 0 ? S.flags[5] : lane < lim ? (int)S.acts[(s + lane) & (kActChunk - 1)] : 0;
+                int goal = cf.ch_goal < 0;
+                if (cf.ch_goal >= 0)
+                    for (int w = lane; w < NW; w += 32)
+                        goal |= S.planes[cf.ch_goal * NWP + w].x != 0u;
+                goal = __any_sync(0xffffffffu, goal);
+                const bool done_l = !goal || (cf.max_steps > 0 && t + lane + 1 >= cf.max_steps);
+                const bool known_l = (S.flags[4] >> a_l) & 1;
+                const uint32_t stop =
+                    __ballot_sync(0xffffffffu, lane < lim && (!known_l || (done_l && cf.auto_reset)));
+                const int e = stop ? __ffs(stop) - 1 : lim;  // steps s .. s + e - 1 repeat the board
+                const int r_l = lane < e ? S.flags[8 + a_l] : 0;
+                if (lane < e) {
+                    if (rew_traj)
+                        rew_traj[(size_t)(s + lane) * cf.B + env] = r_l;
+                    if (done_traj)
+                        done_traj[(size_t)(s + lane) * cf.B + env] = (uint8_t)done_l;
+                }
+                sum += __reduce_add_sync(0xffffffffu, r_l);
+                t += e;
+                a_next = __shfl_sync(0xffffffffu, a_l, e & 31);  // (read from the ring when e = lim)
+                if (e == lim && s + e < n_steps)
+                    a_next = S.acts[(s + e) & (kActChunk - 1)];
+                if (lane == 0)
+                    S.flags[6] = e;
+            }
+            __syncthreads();
+            const int e = S.flags[6];
+            if (e > 0) {
+                if (warp == 0 && s + e < n_steps) {
+                    write_force(cf, S, a_next);
+                    if (lane == 0)
+                        S.flags[5] = a_next;
+                }
+                if (obs_traj)
+                    store_cells_steps<CellT>(cf, S.planes, obs_traj + ((size_t)s * cf.B + env) * HW,
+                                             (size_t)cf.B * HW, e, tid, kThreads);
+                __syncthreads();
+                s += e - 1;
+                continue;
+            }
+        }
         const int a = S.flags[5];
         const bool known = (S.flags[4] >> a) & 1;  // block-uniform (written before the last barrier)
         if (!known)
