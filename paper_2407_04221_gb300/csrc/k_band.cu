@@ -118,9 +118,72 @@ __global__ void __launch_bounds__(kThreads)
     // of S.flags[4], its reward in S.flags[8 + a]) and its later steps skip the
     // bands until the board changes or resets.
     const int n_bands = (H + band_rows - 1) / band_rows;
+    const int warp = tid >> 5, lane = tid & 31;
     for (int s = 0; s < n_steps; ++s) {
-        if (((s + 1) & (kActChunk - 1)) == 0)
+        const bool refill = ((s + 1) & (kActChunk - 1)) == 0;
+        if (refill)
             fill_actions(actions, seed, env, s + 1, n_steps, S);
+        // A run of repeated steps, as in the block rollout: from this step on,
+        // the steps whose actions are remembered and that end no episode with
+        // an auto-reset take their remembered rewards, up to 32 at a time (lane
+        // l of warp 0 takes step s + l), never up to the last step of the action
+        // ring's chunk.  Warp 0 publishes the run's length and the next step's
+        // action (S.flags[6], [7]) before a barrier that every thread reaches
+        // after reading this step's action; the next force plane and S.flags[5]
+        // are written after it, and a second barrier ends the run.
+        if ((S.flags[4] >> S.flags[5]) & 1) {  // block-uniform
+            if (refill)
+                __syncthreads();  // the ring's next chunk
+            if (warp == 0) {
+                const int lim = min(min(32, n_steps - s), ((s + 1) | (kActChunk - 1)) - s);
+                const int a_l = lane == 0 ? S.flags[5] : lane < lim ? (int)S.acts[(s + lane) & (kActChunk - 1)] : 0;
+                const bool done_l = !goal_left || (cf.max_steps > 0 && t + lane + 1 >= cf.max_steps);
+                const bool known_l = (S.flags[4] >> a_l) & 1;
+                const uint32_t stop =
+                    __ballot_sync(0xffffffffu, lane < lim && (!known_l || (done_l && cf.auto_reset)));
+                const int e = stop ? __ffs(stop) - 1 : lim;  // steps s .. s + e - 1 repeat the board
+                const int r_l = lane < e ? S.flags[8 + a_l] : 0;
+                if (lane < e) {
+                    if (rew_traj)
+                        rew_traj[(size_t)(s + lane) * cf.B + env] = r_l;
+                    if (done_traj)
+                        done_traj[(size_t)(s + lane) * cf.B + env] = (uint8_t)done_l;
+                }
+                sum += __reduce_add_sync(0xffffffffu, r_l);  // (thread 0's sum is the one kept)
+                int a_next = __shfl_sync(0xffffffffu, a_l, e & 31);
+                if (e == lim && s + e < n_steps)
+                    a_next = S.acts[(s + e) & (kActChunk - 1)];
+                if (lane == 0) {
+                    S.flags[6] = e;
+                    S.flags[7] = a_next;
+                }
+            }
+            __syncthreads();
+            const int e = S.flags[6];
+            if (e > 0) {
+                t += e;
+                if (s + e < n_steps) {
+                    const int a = S.flags[7];
+                    for (int w = tid; w < NW; w += kThreads)
+                        P[C * NW + w] =
+                            force_word(cf, P + (cf.ch_player >= 0 ? cf.ch_player : 0) * NW, masks_g, NW, w, a);
+                    if (tid == 0)
+                        S.flags[5] = a;
+                }
+                if (obs_traj) {
+                    for (int p = tid; p < HW; p += kThreads) {
+                        uint32_t v = 0;
+                        for (int c = 0; c < C; ++c)
+                            v |= ((P[c * NW + (p >> 5)] >> (p & 31)) & 1u) << c;
+                        for (int k = 0; k < e; ++k)
+                            obs_traj[((size_t)(s + k) * cf.B + env) * HW + p] = (CellT)v;
+                    }
+                }
+                __syncthreads();
+                s += e - 1;
+                continue;
+            }
+        }
         const int act = S.flags[5];
         const bool known = (S.flags[4] >> act) & 1;  // block-uniform (written before the last barrier)
         int rew = 0;

@@ -136,7 +136,8 @@ struct Smem {
     uint32_t *setp, *clrp, *basep, *vm, *masks, *rules;
     int *red, *flags;  // flags: [0] a match this step, [1] action warning, [3] band step reward,
                        // [4] rollout_kernel's remembered actions, [5] its coming step's action,
-                       // [6] its run of repeated steps, [8 + a] the remembered rewards
+                       // [6] the length of a run of repeated steps, [7] the action after a band
+                       // kernel run, [8 + a] the remembered rewards
     uint8_t *acts;
     uint16_t *cells;
 };
