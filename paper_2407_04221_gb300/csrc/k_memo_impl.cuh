@@ -77,7 +77,7 @@ __host__ __device__ inline MemoLayout memo_layout(const DevConfig &cf, bool stag
 
 // Whether the whole rule table is copied into shared memory: when the
 // environment's region with it still lets six environments share an SM (the
-// register budget allows eight); else the table is read through the L1 cache,
+// register budget allows seven); else the table is read through the L1 cache,
 // and only for rules that pass their leading terms.  On the trajectory
 // workload (the largest table 31 KB with its region: seven per SM) staging
 // took the launch from 18.3 to 16.1 ms.  AV_MEMO_STAGE=1 (copy) or 0 (do not),
@@ -536,8 +536,10 @@ __device__ __forceinline__ void memo_cells(const DevConfig &cf, const uint2 *pla
 // Fused rollout, one CTA of NWARP warps per environment; see the top of this
 // file.  With `actions` non-null the action of every step is actions[env]
 // (av_step, n_steps = 1); else step s draws draw(seed, 4, env, 0, s) mod 5.
+// Four warps: 72 registers a thread (seven CTAs per SM, which shared memory
+// allows on the trajectory workload anyway: 13.7 against 14.0 ms at 64).
 template <typename CellT, int NA, bool SM, int NWARP>
-__global__ void __launch_bounds__(32 * NWARP, 32 / NWARP)
+__global__ void __launch_bounds__(32 * NWARP, NWARP == 4 ? 7 : 32 / NWARP)
 rollout_memo_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
                     const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
                     const CellT *__restrict__ init, int32_t *tsteps, int n_steps, uint64_t seed,
