@@ -2,6 +2,8 @@
 // current GPU, for the ALU roofline of the benchmark.  Eight independent
 // dependency chains per thread, 8 CTAs of 256 threads per SM; per-CTA cycles
 // come from clock64, so the rate per clock does not depend on the SM clock.
+// A stand-alone measurement program (`bench.py --int-probe` builds and runs
+// it): not part of libautoverse.so, and nothing in the library calls it.
 #include <cstdio>
 #include <cstdint>
 #include <cuda_runtime.h>
