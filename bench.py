@@ -43,10 +43,12 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "kernels.cuh")
 PROFILE_DIR = os.path.join(ROOT, "profiles")
 # rollout kernel launched for each av_rollout_path value
 KERNEL_NAMES = {1: "rollout_kernel", 2: "rollout_fast_kernel", 3: "rollout_env_warp_kernel",
-                4: "rollout_variant_kernel", 5: "rollout_band_kernel", 6: "rollout_memo_kernel"}
+                4: "rollout_variant_kernel", 5: "rollout_band_kernel", 6: "rollout_memo_kernel",
+                7: "step_warp_kernel"}
 VARIANT_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_variant.cu")
 MEMO_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_memo_impl.cuh")
 BAND_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_band.cu")
+STEP_SRC = os.path.join(ROOT, "paper_2407_04221_gb300", "csrc", "k_step.cu")
 
 
 def bench_variant(wl) -> dict:
@@ -375,10 +377,12 @@ def profile_field(kernel: str, wl, field: str, src=KERNEL_SRC) -> float | None:
 
 
 def kernel_source(path: int, av):
-    """The source of the rollout kernel for an av_rollout_path value: its file,
-    or its files hashed together."""
+    """The source of the rollout kernel for an av_rollout_path (or
+    av_step_path) value: its file, or its files hashed together."""
     if path == av.AV_PATH_MEMO:
         return (MEMO_SRC, KERNEL_SRC)
+    if path == av.AV_PATH_STEP:
+        return (STEP_SRC, KERNEL_SRC)
     if path == av.AV_PATH_VARIANT:
         return VARIANT_SRC
     if path == av.AV_PATH_BAND:
@@ -713,9 +717,7 @@ def run_single_step(args, wl):
 
     if rank == 0:
         peaks = measured_peaks()
-        path = av.av_rollout_path(env.h)
-        if path == av.AV_PATH_MEMO and not os.environ.get("AV_KERNEL_PATH"):
-            path = av.AV_PATH_BLOCK  # av_step's default kernel on small boards
+        path = av.av_step_path(env.h)
         kernel = KERNEL_NAMES[path]
         src = kernel_source(path, av)
         sw = SingleStepName(wl)

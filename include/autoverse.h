@@ -354,12 +354,20 @@ int av_warnings(av_handle *h, uint32_t *bits);
  * most 16 rules) step every environment every step; they run when the
  * environment variable AV_KERNEL_PATH=block|fast|warp|memo, read by av_create,
  * forces a path for tests and measurements.  Every path gives the same
- * results.  The path named is av_rollout's; av_step (one step per launch, no
- * outcome to repeat) takes the block kernel unless AV_KERNEL_PATH forces one.
+ * results.  The path named is av_rollout's; av_step's is av_step_path's.
  * Writes the path to *path; AV_EINVAL for a null argument.  No GPU work. */
 enum { AV_PATH_BLOCK = 1, AV_PATH_FAST = 2, AV_PATH_WARP = 3, AV_PATH_VARIANT = 4, AV_PATH_BAND = 5,
-       AV_PATH_MEMO = 6 };
+       AV_PATH_MEMO = 6, AV_PATH_STEP = 7 };
 int av_rollout_path(av_handle *h, int32_t *path);
+
+/* Which kernel av_step launches for this handle (Sec. 2.1, one step of every
+ * environment given its action): AV_PATH_STEP (one warp per environment,
+ * eight environments per CTA, the rule table read where it lies: boards of at
+ * most 512 cells), AV_PATH_BLOCK (larger boards, up to 64 x 64), or, with
+ * variant semantics set, boards in bands, or AV_KERNEL_PATH forcing a path,
+ * the kernel av_rollout_path names.  Every path gives the same results.
+ * Writes the path to *path; AV_EINVAL for a null argument.  No GPU work. */
+int av_step_path(av_handle *h, int32_t *path);
 
 /* Static description of a status code. */
 const char *av_strerror(int status);

@@ -24,13 +24,14 @@ AV_PATH_BLOCK, AV_PATH_FAST, AV_PATH_WARP = 1, 2, 3
 RULE_BYTES = 408
 EXPORTS = ("av_create", "av_destroy", "av_reset", "av_set_state", "av_get_state", "av_step",
            "av_rollout", "av_expand", "av_search_init", "av_select", "av_select_static", "av_sync",
-           "av_warnings", "av_rollout_path", "av_observe", "av_rule_obs", "av_mutate", "av_set_variant", "av_strerror",
+           "av_warnings", "av_rollout_path", "av_step_path", "av_observe", "av_rule_obs", "av_mutate", "av_set_variant", "av_strerror",
            "av_last_error")
 AV_MAX_WINDOW = 127
 AV_MAX_LIMIT = 255
 AV_PATH_VARIANT = 4
 AV_PATH_BAND = 5
 AV_PATH_MEMO = 6
+AV_PATH_STEP = 7
 AV_MAX_SMEM_CELLS = 4096
 AV_SELECT_STATIC_MAX_HASHES = 1 << 21
 
@@ -94,6 +95,7 @@ def load() -> ctypes.CDLL:
         "av_sync": [vp],
         "av_warnings": [vp, ctypes.POINTER(ctypes.c_uint32)],
         "av_rollout_path": [vp, ctypes.POINTER(ctypes.c_int32)],
+        "av_step_path": [vp, ctypes.POINTER(ctypes.c_int32)],
         "av_observe": [vp, vp, i32, vp, vp, up],
         "av_rule_obs": [vp, vp, vp, up],
         "av_mutate": [i32, i32, i32, i32, i32, ctypes.POINTER(AvMutation), u64, vp, vp, up],
@@ -246,6 +248,12 @@ def av_warnings(h) -> int:
 def av_rollout_path(h) -> int:
     path = ctypes.c_int32()
     _check(h, "av_rollout_path", load().av_rollout_path(h, ctypes.byref(path)))
+    return int(path.value)
+
+
+def av_step_path(h) -> int:
+    path = ctypes.c_int32()
+    _check(h, "av_step_path", load().av_step_path(h, ctypes.byref(path)))
     return int(path.value)
 
 

@@ -11,7 +11,7 @@ LIB = os.path.join(PKG, "libautoverse.so")
 SOURCES = [os.path.join(CSRC, f) for f in ("autoverse.cu", "k_fast_u8.cu", "k_fast_u16.cu", "k_warp_u8.cu",
                                             "k_warp_u16.cu", "k_block.cu", "k_expand.cu", "k_search.cu",
                                             "k_observe.cu", "k_mutate.cu", "k_memo_u8.cu", "k_memo_u16.cu",
-                                            "k_variant.cu", "k_band.cu")]
+                                            "k_variant.cu", "k_band.cu", "k_step.cu")]
 DEPS = SOURCES + [os.path.join(CSRC, f) for f in ("kernels.cuh", "launch.h", "k_fast_impl.cuh", "k_warp_impl.cuh",
                                                      "k_memo_impl.cuh")] + [
     os.path.join(ROOT, "include", "autoverse.h")]

@@ -1014,6 +1014,17 @@ int av_rollout_path(av_handle *h, int32_t *path)
     return AV_OK;
 }
 
+int av_step_path(av_handle *h, int32_t *path)
+{
+    AV_HANDLE(h);
+    if (!h || !path)
+        return AV_EINVAL;
+    if (h->large || h->variant_on || h->cf.path != 0)
+        return av_rollout_path(h, path);  // av_step takes av_rollout's kernel
+    *path = use_step_warp(h->cf) ? AV_PATH_STEP : AV_PATH_BLOCK;
+    return AV_OK;
+}
+
 int av_warnings(av_handle *h, uint32_t *bits)
 {
     AV_HANDLE(h);

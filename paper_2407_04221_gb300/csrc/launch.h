@@ -21,6 +21,14 @@ cudaError_t configure_search();
 cudaError_t configure_observe();
 cudaError_t configure_memo_u8();
 cudaError_t configure_memo_u16();
+cudaError_t configure_step();
+
+// One step of every environment given its action, one warp per environment
+// (k_step.cu): av_step's kernel for boards of at most 16 plane words.
+bool use_step_warp(const DevConfig &cf);
+void launch_step_warp(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off, const uint32_t *vm,
+                      const uint32_t *masks, void *cur, const void *init, int32_t *t, const uint8_t *actions,
+                      void *obs, int32_t *rew, uint8_t *done, int32_t *rew_sum, uint32_t *status, cudaStream_t st);
 
 void launch_rollout_fast_u8(const DevConfig &cf, const uint32_t *arena, const uint32_t *tab_off,
                             const uint32_t *vm, const uint32_t *masks, void *cur, const void *init,
@@ -130,6 +138,7 @@ inline cudaError_t configure_kernels()
     if (e == cudaSuccess) e = configure_observe();
     if (e == cudaSuccess) e = configure_memo_u8();
     if (e == cudaSuccess) e = configure_memo_u16();
+    if (e == cudaSuccess) e = configure_step();
     if (e == cudaSuccess) e = configure_variant();
     if (e == cudaSuccess) e = configure_band();
     return e;
@@ -142,12 +151,15 @@ inline void launch_rollout(const DevConfig &cf, const uint32_t *arena, const uin
                            cudaStream_t st, const int32_t *order = nullptr, uint32_t *cost = nullptr)
 {
     // A launch of one step given its actions (av_step) has no outcome to
-    // repeat: by default it takes the block kernel, whose setup is the
-    // shortest (measured on the 16,384-env training shape: 0.126 ms against
-    // 0.147-0.184 ms for the memoising kernel).
+    // repeat: by default it takes the one-warp step kernel (small boards) or
+    // the block kernel, whose setups are the shortest.
     if (n_steps == 1 && actions && cf.path == 0) {
-        launch_rollout_block(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
-                             rew_traj, done_traj, rew_sum, status, st);
+        if (use_step_warp(cf))
+            launch_step_warp(cf, arena, tab_off, vm, masks, cur, init, t, actions, obs_traj, rew_traj, done_traj,
+                             rew_sum, status, st);
+        else
+            launch_rollout_block(cf, arena, tab_off, vm, masks, cur, init, t, n_steps, seed, actions, obs_traj,
+                                 rew_traj, done_traj, rew_sum, status, st);
         return;
     }
     if (use_memo_rollout(cf) && cf.cell_bytes == 1)

@@ -2,7 +2,9 @@
 
 All 4^9 = 262,144 boards of a 3 x 3 grid whose cells hold any subset of two
 tile channels (channel 0 the player, channel 1 the goal), each stepped with
-each of the five actions by `av_step` on every rollout kernel, compared with
+each of the five actions by `av_step` on every kernel (the one-warp step
+kernel that `av_step` takes by default, and every rollout kernel forced by
+AV_KERNEL_PATH), compared with
 the oracle element by element: boards, rewards and done flags.  The rule
 tables are the ones whose oracle step is pinned against the convolution
 formulation of Sec. 2.1 (Eq. 1 and Eq. 3) on the same enumeration in
@@ -25,7 +27,7 @@ from tests.gpu_helpers import to_dev, to_np
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-PATHS = ["block", "fast", "fast8", "warp", "memo", "variant-warp", "variant-block"]
+PATHS = ["step", "block", "fast", "fast8", "warp", "memo", "variant-warp", "variant-block"]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -77,11 +79,14 @@ def test_every_3x3_board_every_action(monkeypatch, path, rule_seed):
     import paper_2407_04221_gb300 as av
     boards, rules, fields, per_action = _expected(rule_seed)
     kernel = path.split("-")[-1]
-    monkeypatch.setenv("AV_KERNEL_PATH", kernel.rstrip("8"))
+    if kernel != "step":
+        monkeypatch.setenv("AV_KERNEL_PATH", kernel.rstrip("8"))
     if kernel.endswith("8"):
         monkeypatch.setenv("AV_FAST_WARPS", "8")
     env = av.Env(fields, rules)
-    if path.startswith("variant"):
+    if kernel == "step":
+        assert av.av_step_path(env.h) == av.AV_PATH_STEP
+    elif path.startswith("variant"):
         av.av_set_variant(env.h, random_keys=0, limit=[255] * 4, inhibit=[0] * 4)
         assert av.av_rollout_path(env.h) == av.AV_PATH_VARIANT
     else:

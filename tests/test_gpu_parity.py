@@ -163,6 +163,8 @@ def test_step_random_actions(key):
     import paper_2407_04221_gb300 as av
     wl = wk.WORKLOADS[key].scaled(batch=33 if key != 5 else 4, max_steps=6, auto_reset=1)
     env, cfg, rules, cum = make(wl, 3)
+    # one warp per environment for 16 x 16 boards, the block kernel for 64 x 64
+    assert av.av_step_path(env.h) == (av.AV_PATH_BLOCK if key == 5 else av.AV_PATH_STEP)
     g0 = to_np(env.reset(77))
     rng = np.random.default_rng(key)
     cur, t = g0.copy(), np.zeros(wl.batch, np.int32)
