@@ -23,8 +23,8 @@ namespace {
 constexpr int kStepWarps = 8;  // environments per CTA
 
 struct StepWarpLayout {
-    size_t vm, masks, warps;          // CTA region
-    size_t planes, setp, clrp, per_warp;  // within a warp's region
+    size_t vm, masks, warps;                   // CTA region
+    size_t planes, setp, clrp, hdr, per_warp;  // within a warp's region
     size_t total;
 };
 
@@ -39,7 +39,8 @@ __host__ __device__ inline StepWarpLayout step_warp_layout(const DevConfig &cf)
     L.planes = 0;
     L.setp = align16s((size_t)(cf.C + 2) * cf.NWP * 8);
     L.clrp = align16s(L.setp + (size_t)cf.C * cf.NW * 4);
-    L.per_warp = align16s(L.clrp + (size_t)cf.C * cf.NW * 4);
+    L.hdr = align16s(L.clrp + (size_t)cf.C * cf.NW * 4);
+    L.per_warp = align16s(L.hdr + (size_t)cf.R * 32);
     L.total = L.warps + (size_t)kStepWarps * L.per_warp;
     return L;
 }
@@ -149,9 +150,10 @@ __device__ __forceinline__ void step_load_planes(const DevConfig &cf, const Cell
     }
 }
 
-// Eight CTAs of eight warps per SM: 32 registers a thread.
+// Six CTAs of eight warps per SM: 40 registers a thread (at 32 it spills and
+// runs 6 % slower on the training shape).
 template <typename CellT, int NA>
-__global__ void __launch_bounds__(32 * kStepWarps, 8)
+__global__ void __launch_bounds__(32 * kStepWarps, 6)
 step_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_t *__restrict__ tab_off,
                  const uint32_t *__restrict__ vm_g, const uint32_t *__restrict__ masks_g, CellT *cur,
                  const CellT *__restrict__ init, int32_t *tsteps, const uint8_t *__restrict__ actions,
@@ -171,6 +173,7 @@ step_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_
     uint2 *planes = reinterpret_cast<uint2 *>(wr + L.planes);
     uint32_t *setp = reinterpret_cast<uint32_t *>(wr + L.setp);
     uint32_t *clrp = reinterpret_cast<uint32_t *>(wr + L.clrp);
+    uint4 *hdr = reinterpret_cast<uint4 *>(wr + L.hdr);  // [R][2] the rule headers, copied
     for (int i = lane; i < (C + 2) * NWP; i += 32)
         planes[i] = make_uint2(0u, 0u);
     for (int i = lane; i < C * NW; i += 32) {
@@ -191,17 +194,20 @@ step_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_
     force_plane(cf, planes, masks, a);
     __syncwarp();
 
-    // ---- every rule in its four rotations
+    // ---- every rule in its four rotations (headers copied in one pass, so a
+    // rule's first terms wait on one load from L2 instead of two)
     const int table = cf.rules_per_env ? env : 0;
     const uint32_t *tab = arena + tab_off[table];
+    for (int i = lane; i < 2 * cf.R; i += 32)
+        hdr[i] = __ldg(reinterpret_cast<const uint4 *>(tab + 4) + i);
+    __syncwarp();
     const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
     const uint4 *outs = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, __ldg(tab + 1)));
     const uint32_t pbase = (uint32_t)__cvta_generic_to_shared(planes) + q * 8;
     const uint2 pass = make_uint2((uint32_t)(C + 1) * NWP * 8, kTermAbsent);  // the zero plane, read as absent
     int rew = 0;
     for (int r = 0; r < cf.R; ++r) {
-        const uint4 h0 = __ldg(reinterpret_cast<const uint4 *>(tab + 4 + 8 * r));
-        const uint4 h1 = __ldg(reinterpret_cast<const uint4 *>(tab + 8 + 8 * r));
+        const uint4 h0 = hdr[2 * r], h1 = hdr[2 * r + 1];
         const uint32_t *vmr = vm + ((h1.z >> (8 * g)) & 0xffu) * NW;
         uint32_t m[NA];
         uint32_t any = 0;
