@@ -24,7 +24,7 @@ constexpr int kStepWarps = 8;  // environments per CTA
 
 struct StepWarpLayout {
     size_t vm, masks, warps;                   // CTA region
-    size_t planes, setp, clrp, hdr, per_warp;  // within a warp's region
+    size_t planes, setp, clrp, hdr, lead, per_warp;  // within a warp's region
     size_t total;
 };
 
@@ -40,7 +40,8 @@ __host__ __device__ inline StepWarpLayout step_warp_layout(const DevConfig &cf)
     L.setp = align16s((size_t)(cf.C + 2) * cf.NWP * 8);
     L.clrp = align16s(L.setp + (size_t)cf.C * cf.NW * 4);
     L.hdr = align16s(L.clrp + (size_t)cf.C * cf.NW * 4);
-    L.per_warp = align16s(L.hdr + (size_t)cf.R * 32);
+    L.lead = align16s(L.hdr + (size_t)cf.R * 32);
+    L.per_warp = align16s(L.lead + (size_t)cf.R * 4 * 4 * 8);
     L.total = L.warps + (size_t)kStepWarps * L.per_warp;
     return L;
 }
@@ -173,7 +174,8 @@ step_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_
     uint2 *planes = reinterpret_cast<uint2 *>(wr + L.planes);
     uint32_t *setp = reinterpret_cast<uint32_t *>(wr + L.setp);
     uint32_t *clrp = reinterpret_cast<uint32_t *>(wr + L.clrp);
-    uint4 *hdr = reinterpret_cast<uint4 *>(wr + L.hdr);  // [R][2] the rule headers, copied
+    uint4 *hdr = reinterpret_cast<uint4 *>(wr + L.hdr);     // [R][2] the rule headers, copied
+    uint2 *lead = reinterpret_cast<uint2 *>(wr + L.lead);  // [R][4 rotations][4] first term descriptors
     for (int i = lane; i < (C + 2) * NWP; i += 32)
         planes[i] = make_uint2(0u, 0u);
     for (int i = lane; i < C * NW; i += 32) {
@@ -194,17 +196,24 @@ step_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_
     force_plane(cf, planes, masks, a);
     __syncwarp();
 
-    // ---- every rule in its four rotations (headers copied in one pass, so a
-    // rule's first terms wait on one load from L2 instead of two)
+    // ---- every rule in its four rotations.  The headers, then every rule's
+    // first four term descriptors, are copied in two passes, so that a rule
+    // that fails its first four terms (most do) waits on no load from L2.
     const int table = cf.rules_per_env ? env : 0;
     const uint32_t *tab = arena + tab_off[table];
+    const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+    const uint2 pass = make_uint2((uint32_t)(C + 1) * NWP * 8, kTermAbsent);  // the zero plane, read as absent
     for (int i = lane; i < 2 * cf.R; i += 32)
         hdr[i] = __ldg(reinterpret_cast<const uint4 *>(tab + 4) + i);
     __syncwarp();
-    const uint2 *terms = reinterpret_cast<const uint2 *>(tab + table_terms_word(cf.R));
+    for (int i = lane; i < 16 * cf.R; i += 32) {  // i = (rule, rotation, term)
+        const int r = i >> 4, rot = (i >> 2) & 3, j = i & 3;
+        const uint4 h0 = hdr[2 * r], h1 = hdr[2 * r + 1];
+        lead[i] = (uint32_t)j < h0.x + h0.y ? __ldg(terms + (size_t)(h1.x + j) * 4 + rot) : pass;
+    }
+    __syncwarp();
     const uint4 *outs = reinterpret_cast<const uint4 *>(tab + table_outs_word(cf.R, __ldg(tab + 1)));
     const uint32_t pbase = (uint32_t)__cvta_generic_to_shared(planes) + q * 8;
-    const uint2 pass = make_uint2((uint32_t)(C + 1) * NWP * 8, kTermAbsent);  // the zero plane, read as absent
     int rew = 0;
     for (int r = 0; r < cf.R; ++r) {
         const uint4 h0 = hdr[2 * r], h1 = hdr[2 * r + 1];
@@ -222,9 +231,18 @@ step_warp_kernel(DevConfig cf, const uint32_t *__restrict__ arena, const uint32_
         bool live = __any_sync(0xffffffffu, any != 0u);
         for (uint32_t t = 0; live && t < nt; t += 4) {
             uint2 d[4];
+            if (t == 0) {  // the copied first four
+                const uint4 *lp = reinterpret_cast<const uint4 *>(lead + (r * 4 + g) * 4);
+                const uint4 x = lp[0], y = lp[1];
+                d[0] = make_uint2(x.x, x.y);
+                d[1] = make_uint2(x.z, x.w);
+                d[2] = make_uint2(y.x, y.y);
+                d[3] = make_uint2(y.z, y.w);
+            } else {
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-                d[j] = t + j < nt ? __ldg(tp + 4 * (t + j)) : pass;
+                for (int j = 0; j < 4; ++j)
+                    d[j] = t + j < nt ? __ldg(tp + 4 * (t + j)) : pass;
+            }
             any = 0;
 #pragma unroll
             for (int u = 0; u < NA; ++u) {
