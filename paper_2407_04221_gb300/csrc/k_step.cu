@@ -59,8 +59,11 @@ __device__ __forceinline__ void step_write(const DevConfig &cf, const uint4 *op,
                                            const uint32_t (&m)[NA], uint32_t *wset, uint32_t *wclr)
 {
     const int lane = threadIdx.x & 31, g = lane >> 3, q = lane & 7;
+    uint4 next = n_out ? __ldg(op) : make_uint4(0u, 0u, 0u, 0u);
     for (uint32_t o = 0; o < n_out; ++o) {
-        const uint4 ov = __ldg(op + 4 * o);
+        const uint4 ov = next;
+        if (o + 1 < n_out)  // the next entry's load overlaps this one's work
+            next = __ldg(op + 4 * (o + 1));
         const int d = (int)ov.x;
         const uint32_t sh = ov.y;
         uint32_t cw[NA];
