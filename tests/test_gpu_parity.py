@@ -213,6 +213,46 @@ def test_edge_shapes(H, W, C, shapes, R):
     env.close()
 
 
+@pytest.mark.parametrize("H,W,C,shapes,R,per_env", [
+    (1, 1, 1, ((1, 1),), 2, 1),
+    (3, 5, 2, ((1, 2), (2, 3)), 3, 1),
+    (7, 9, 3, ((3, 3), (5, 5), (1, 4)), 4, 0),   # ragged, rules wider than the board, one shared table
+    (5, 5, 16, ((5, 5), (4, 2)), 2, 1),          # two-byte cells, 17 channels
+    (20, 21, 5, ((3, 3), (2, 5)), 6, 1),         # 420 cells: two anchor words per lane
+    (16, 32, 10, ((3, 3), (1, 3)), 12, 1),       # 512 cells, the largest board of the one-warp step
+    (2, 64, 9, ((1, 5), (2, 2)), 3, 0),
+    (16, 16, 4, ((3, 3),), 0, 1),                # no rules
+])
+def test_step_edge_shapes(H, W, C, shapes, R, per_env):
+    """av_step on its one-warp kernel over ragged and edge board shapes, one and
+    two anchor words per lane, shared and per-environment tables, no rules:
+    six steps of random actions with auto-reset, against the oracle."""
+    import paper_2407_04221_gb300 as av
+    n = 19
+    wl = wk.Workload(0, "edge-step", n, H, W, C, R, shapes, 0.1, 0.06, 0.2, 0.2, -2, 2,
+                     max_steps=4, auto_reset=1, rules_per_env=per_env)
+    _, rules, _ = wk.make(wl, 6)
+    g0 = wk.random_grids(11, n, H, W, C, density=0.4)
+    if C > 2:
+        g0[:, H // 2, W // 2] |= 1 << 2
+    env, cfg, _, _ = make(wl, 0, rules=rules, cum=None)
+    assert av.av_step_path(env.h) == av.AV_PATH_STEP
+    env.set_state(to_dev(g0), set_as_init=True)
+    cur, t = g0.copy(), np.zeros(n, np.int32)
+    rng = np.random.default_rng(H * 100 + W)
+    for _ in range(6):
+        acts = rng.integers(0, 5, n).astype(np.uint8)
+        obs, rew, done = env.step(to_dev(acts))
+        cur, t, erew, edone = oracle.step(cfg, rules, cur, g0, t, acts)
+        np.testing.assert_array_equal(to_np(obs), cur)
+        np.testing.assert_array_equal(to_np(rew), erew)
+        np.testing.assert_array_equal(to_np(done), edone)
+    g, tt = env.get_state()
+    np.testing.assert_array_equal(to_np(g), cur)
+    np.testing.assert_array_equal(to_np(tt), t)
+    env.close()
+
+
 def test_shared_rules_and_zero_rules():
     wl = wk.WORKLOADS[1].scaled(batch=40)  # one shared table, 40 envs
     env, cfg, rules, cum = make(wl, 2)
