@@ -143,7 +143,9 @@ int av_get_state(av_handle *h, void *grids, int32_t *t, uintptr_t stream);
 
 /* One batched step (Sec. 2.1): actions device uint8[B]; obs device
  * [B][H][W] or NULL; reward device int32[B]; done device uint8[B] (reward
- * and done may be NULL).  Updates the handle's boards and t. */
+ * and done may be NULL).  Updates the handle's boards and t.  An action
+ * above 4 acts as 0 and sets AV_WARN_ACTION.  av_step_path names the kernel
+ * it launches (one warp per environment for boards of at most 512 cells). */
 int av_step(av_handle *h, const uint8_t *actions, void *obs, int32_t *reward, uint8_t *done,
             uintptr_t stream);
 
