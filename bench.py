@@ -726,6 +726,8 @@ def run_single_step(args, wl):
         peak = float(peaks.get("hbm_gbs", 6723.0))
         achieved = bpes * wl.batch / (kernel_ms / 1e3) / 1e9
         traffic = profile_traffic(kernel, sw, src)
+        inst = profile_field(kernel, sw, "warp_instructions_per_launch", src)
+        clock = float((clocks or {}).get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)) * 1e6
         line = {
             "metric": "env-steps/s", "value": value, "unit": "env-steps/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
@@ -744,7 +746,12 @@ def run_single_step(args, wl):
                                         " the env's rule table (per-env tables, read every launch)"
                                         " are extra traffic, counted in `traffic`",
                          "traffic_per_env_step": traffic / wl.batch if traffic else None,
-                         "peak_from": "hbm_gbs of measured peaks (copy bandwidth)"},
+                         "peak_from": "hbm_gbs of measured peaks (copy bandwidth)",
+                         "issue_util": (inst / (SM_COUNT_GB300 * 4 * clock * kernel_ms / 1e3))
+                                       if inst else None,
+                         "issue_util_basis": "ncu warp instructions of one launch (committed"
+                                             " profile) / (152 SMs x 4 schedulers x median SM"
+                                             " clock x launch time): the step's limiter"},
             "gpu_launches": args.steps,
             "wall_s_timed_region": wall,
         }
